@@ -1,0 +1,412 @@
+#!/usr/bin/env python
+"""Benchmark of the Similarity Chunk Rolling sparse-prefill path on GB300.
+
+One step = steps (a)-(d) of the path over one layer of the workload: block
+representatives + fingerprints + anchor clusters, cluster-level selection,
+block-sparse causal attention. Inputs are resident in HBM before timing; they
+are larger than L2 (Q, K, V of the 128K workload are 1.6 GB).
+
+Prints one JSON line (rank 0). ``--impl reference`` times the CPU fp64 oracle
+instead, on a bounded sample of the same workload.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from synth import generate_layer, workload  # noqa: E402
+
+METRIC = "sparse-prefill tokens/sec and TTFT at 128K ctx on 1 GB300; % of roofline"
+DEFAULT_WORKLOAD = "llama8b-128k"
+KERNEL_SRC = os.path.join(ROOT, "paper_2609_31568_gb300", "csrc", "attn.cu")
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "attn_llama8b-128k_ncu.md")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["scale", "reference"], default="scale")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--mode", choices=["cluster", "subchunk"], default="cluster")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-baseline-mode", action="store_true",
+                    help="skip timing the per-sub-chunk selection mode alongside")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="target CPU time of the oracle sample")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------------------- helpers
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            pk = json.load(f)
+        return dict(hbm=pk.get("hbm_gbs", 6800.0), bf16=pk.get("bf16_tflops", 1900.0),
+                    bf16_sustained=pk.get("bf16_tflops_sustained", 1700.0), source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
+
+
+def key_counts(w, unit_start, n_units, sel, cnt, per_subchunk):
+    """Sum over query rows of |K(p)|, the distinct keys each row attends to (Eq. 10)."""
+    total = 0
+    for u in range(n_units):
+        a = u if per_subchunk else int(unit_start[u])
+        b = u + 1 if per_subchunk else int(unit_start[u + 1])
+        s, e = a * w.sub_chunk, min(w.n_tokens, b * w.sub_chunk)
+        W = max(0, s - w.n_local)
+        D = min(w.n_sink, W)
+        for blk in sel[u, : int(cnt[u])]:
+            lo = max(int(blk) * w.block_size, w.n_sink)
+            hi = min((int(blk) + 1) * w.block_size, W)
+            D += max(0, hi - lo)
+        n = e - s
+        total += n * D + n * (s - W + 1) + n * (n - 1) // 2
+    return total
+
+
+def profile_traffic():
+    """Per-launch DRAM bytes of the attention kernel from the committed ncu
+    summary, or None when the kernel source changed since the capture."""
+    if not os.path.exists(PROFILE_SUMMARY):
+        return None
+    with open(KERNEL_SRC, "rb") as f:
+        sha = hashlib.sha256(f.read()).hexdigest()[:16]
+    vals = {}
+    with open(PROFILE_SUMMARY) as f:
+        for line in f:
+            if ":" in line and line.strip().startswith("- "):
+                k, v = line.strip()[2:].split(":", 1)
+                vals[k.strip()] = v.strip()
+    if vals.get("attn.cu sha256[:16]") != sha:
+        return None
+    try:
+        return float(vals["traffic bytes per full launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int = 0):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            import torch
+
+            uuid = str(torch.cuda.get_device_properties(self.dev).uuid)
+            sel = ["-i", uuid if uuid.startswith("GPU-") else "GPU-" + uuid]
+        except Exception:
+            sel = ["-i", str(self.dev)]
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", *sel, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.4)
+        except FileNotFoundError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, val in zip(names, parts[5:9]):
+                    if val.lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- oracle timing
+
+
+def oracle_sample(w, q, k, v, per_subchunk, cpu_seconds, rows_first=32):
+    """Time the oracle on a bounded sample: steps (a)-(c) over the whole layer,
+    step (d) on a growing set of seeded rows until about cpu_seconds; the
+    throughput is extrapolated from the per-row time to all rows."""
+    import oracle
+
+    t0 = time.perf_counter()
+    ref = oracle.run_path(w, q, k, v, per_subchunk=per_subchunk)
+    t_abc = time.perf_counter() - t0
+    rng = np.random.default_rng(7)
+    n_rows, t_d, done = rows_first, 0.0, 0
+    while True:
+        rows = np.sort(rng.integers(0, w.n_tokens, size=n_rows))
+        t1 = time.perf_counter()
+        oracle.attention_rows(q=q, k=k, v=v, sub_chunk=w.sub_chunk, block_size=w.block_size,
+                              top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                              attn_scale=1.0 / np.sqrt(w.head_dim), per_subchunk=per_subchunk,
+                              unit_start=ref["unit_start"], sel=ref["sel"],
+                              sel_count=ref["sel_count"], rows=rows)
+        t_d += time.perf_counter() - t1
+        done += n_rows
+        if t_abc + t_d >= cpu_seconds or done >= w.n_tokens:
+            break
+        n_rows = min(w.n_tokens, max(n_rows, int(n_rows * max(1.5, (cpu_seconds - t_abc) / max(t_d, 1e-3) * 0.6))))
+    t_full = t_abc + t_d / done * w.n_tokens
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    omp = os.environ.get("OMP_NUM_THREADS")
+    return dict(tokens_per_s=w.n_tokens / t_full, t_full=t_full, t_abc=t_abc, t_d=t_d, rows=done,
+                cores=int(omp) if omp else cores)
+
+
+# --------------------------------------------------------------------------- arms
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_reference(args):
+    world, rank, local = dist_setup(args)
+    if rank != 0:
+        return 0
+    w = workload(args.workload)
+    per_sub = args.mode == "subchunk"
+    q, k, v = generate_layer(w)
+    times, last = [], None
+    for i in range(args.warmup + args.steps):
+        r = oracle_sample(w, q, k, v, per_sub, cpu_seconds=max(1.0, args.cpu_seconds / 4), rows_first=16)
+        if i >= args.warmup:
+            times.append(r["t_full"])
+            last = r
+    t = statistics.mean(times)
+    value = w.n_tokens / t
+    sample = (f"per step: steps (a)-(c) over all {w.n_tokens} tokens ({last['t_abc']:.2f} s) + "
+              f"Eq. 10 on {last['rows']} seeded rows ({last['t_d']:.2f} s), extrapolated per row")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": w.name, "n_tokens": w.n_tokens, "mode": args.mode, "theta": w.theta},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": last["cores"], "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_scale(args):
+    import torch
+
+    world, rank, local = dist_setup(args)
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    import paper_2609_31568_gb300 as pkg
+    from paper_2609_31568_gb300 import scale as S
+
+    pkg.build()
+    S.load()
+    w = workload(args.workload)
+    mode = S.SCALE_MODE_PER_SUBCHUNK if args.mode == "subchunk" else S.SCALE_MODE_PER_CLUSTER
+    per_sub = mode == S.SCALE_MODE_PER_SUBCHUNK
+    # weak scaling: every rank prefills its own independent layer (seed + rank)
+    q, k, v = generate_layer(w, seed=w.seed + rank)
+    dev = [torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)]
+    p = S.params_for(w)
+    buf = pkg.allocate(p, mode)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    def timed(mode_, steps, warmup, buf_):
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
+        for _ in range(warmup):
+            pkg.run_path(p, mode_, *dev, buf_)
+        torch.cuda.synchronize()
+        barrier()
+        torch.cuda.synchronize()
+        clocks = ClockSampler(torch.cuda.current_device())
+        clocks.start()
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for i in range(steps):
+            e = ev[i]
+            e[0].record(stream)
+            S.scale_build_reps(p, dev[0], dev[1], buf_.reps, buf_.fingerprints, buf_.unit_start,
+                               buf_.n_units, buf_.ws, stream)
+            e[1].record(stream)
+            S.scale_select(p, mode_, 0, w.n_tokens, buf_.reps, buf_.fingerprints, buf_.unit_start,
+                           buf_.n_units, buf_.sel_blocks, buf_.sel_count, None, buf_.ws, stream)
+            e[2].record(stream)
+            S.scale_sparse_prefill(p, mode_, 0, w.n_tokens, *dev, buf_.unit_start, buf_.n_units,
+                                   buf_.sel_blocks, buf_.sel_count, buf_.out, buf_.ws, stream)
+            e[3].record(stream)
+        end.record(stream)
+        torch.cuda.synchronize()
+        clk = clocks.stop()
+        barrier()
+        total = start.elapsed_time(end) / steps
+        stages = [statistics.mean(x[j].elapsed_time(x[j + 1]) for x in ev) for j in range(3)]
+        st = S.scale_get_device_status(buf_.ws)
+        if st != S.SCALE_OK:
+            raise RuntimeError(f"device status {st}: {S.status_string(st)}")
+        return total, stages, clk
+
+    ms, stages, clk = timed(mode, args.steps, args.warmup, buf)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+
+    n_units = w.n_subchunks if per_sub else int(buf.n_units.item())
+    us = buf.unit_start.cpu().numpy()
+    sel = buf.sel_blocks.cpu().numpy()
+    cnt = buf.sel_count.cpu().numpy()
+    keys = key_counts(w, us, n_units, sel, cnt, per_sub)
+    flops = 4.0 * w.head_dim * w.num_q_heads * keys
+    peaks = load_peaks()
+    attn_s = stages[2] / 1e3
+    achieved = flops / attn_s / 1e12
+    _, calls = S.scale_retrieval_calls(p, mode, us[: n_units + 1] if not per_sub else None, n_units)
+
+    line = {
+        "metric": METRIC,
+        "value": world * w.n_tokens / (ms / 1e3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms,
+        "ttft_ms": ms,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": w.name, "n_tokens": w.n_tokens, "q_heads": w.num_q_heads,
+                   "kv_heads": w.num_kv_heads, "head_dim": w.head_dim, "sub_chunk": w.sub_chunk,
+                   "max_cluster_subchunks": w.max_cluster_subchunks, "block_size": w.block_size,
+                   "top_k": w.top_k, "n_sink": w.n_sink, "n_local": w.n_local, "theta": w.theta,
+                   "mode": args.mode, "parallelism": f"independent layers x{world}",
+                   "l2": "inputs larger than L2 (Q+K+V %.2f GB)" % ((q.nbytes + k.nbytes + v.nbytes) / 1e9)},
+        "stages_ms": {"build_reps": stages[0], "select": stages[1], "sparse_attention": stages[2]},
+        "retrieval_calls": calls,
+        "units": n_units,
+        "roofline": {"bound": "tensor", "kernel": "k_sparse_attn", "achieved": achieved,
+                     "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
+                     "frac": achieved / peaks["bf16_sustained"],
+                     "frac_of_burst": achieved / peaks["bf16"],
+                     "peak_source": f"bf16 sustained, of {peaks['source']}",
+                     "algorithmic_flops_per_launch": flops, "traffic": profile_traffic()},
+        "gpu_launches": args.steps * (10 if w.max_cluster_subchunks > 1 else 9),
+        "clocks": clk,
+    }
+
+    if not args.no_baseline_mode and rank == 0:
+        other = S.SCALE_MODE_PER_SUBCHUNK if not per_sub else S.SCALE_MODE_PER_CLUSTER
+        buf2 = pkg.allocate(p, other)
+        ms2, st2, _ = timed(other, max(3, args.steps // 2), 2, buf2)
+        n2 = w.n_subchunks if other == S.SCALE_MODE_PER_SUBCHUNK else int(buf2.n_units.item())
+        us2 = buf2.unit_start.cpu().numpy()
+        _, calls2 = S.scale_retrieval_calls(
+            p, other, us2[: n2 + 1] if other == S.SCALE_MODE_PER_CLUSTER else None, n2)
+        line["other_mode"] = {"mode": "subchunk" if other == S.SCALE_MODE_PER_SUBCHUNK else "cluster",
+                              "ms_per_step": ms2, "tokens_per_s": w.n_tokens / (ms2 / 1e3),
+                              "stages_ms": {"build_reps": st2[0], "select": st2[1], "sparse_attention": st2[2]},
+                              "retrieval_calls": calls2, "units": n2}
+        del buf2
+
+    if not args.no_e2e:
+        qh, kh, vh = (torch.from_numpy(x).pin_memory() for x in (q, k, v))
+        oh = torch.empty(qh.shape, dtype=torch.int16).pin_memory()
+        arena = torch.empty(S.scale_prefill_host_arena_size(p, mode), dtype=torch.uint8, device="cuda")
+        S.scale_prefill_host(p, mode, qh, kh, vh, oh, arena, stream)
+        reps = max(3, args.steps // 4)
+        torch.cuda.synchronize()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            S.scale_prefill_host(p, mode, qh, kh, vh, oh, arena, stream)
+        t_e2e = (time.perf_counter() - t0) / reps
+        if world > 1:
+            t = torch.tensor([t_e2e], device="cuda")
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            t_e2e = float(t.item())
+        line["e2e"] = {"value": world * w.n_tokens / t_e2e, "unit": "tokens/s",
+                       "h2d_bytes_per_step": int(q.nbytes + k.nbytes + v.nbytes),
+                       "d2h_bytes_per_step": int(q.nbytes), "ms_per_step": t_e2e * 1e3,
+                       "api": "scale_prefill_host (pinned host buffers)"}
+        del arena
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        r = oracle_sample(w, q, k, v, per_sub, args.cpu_seconds)
+        line["cpu_baseline"] = {
+            "value": r["tokens_per_s"], "unit": "tokens/s", "cores": r["cores"], "kind": "oracle",
+            "sample": (f"steps (a)-(c) over all {w.n_tokens} tokens ({r['t_abc']:.2f} s) + Eq. 10 on "
+                       f"{r['rows']} seeded rows ({r['t_d']:.2f} s), time per row extrapolated to all rows")}
+
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_scale(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,201 @@
+/*
+ * scale.h -- C ABI of libscale, a GB300 (sm_103a) implementation of the
+ * prefill hot path of Similarity Chunk Rolling (SCR), the long-context engine
+ * of SCALE (arXiv 2609.31568, Sec. V-A).
+ *
+ * SCR runs chunked prefill with selective sparse attention (Sec. III-B, Def. 1,
+ * Eq. 3-4) and performs the selection once per *cluster* of similar query
+ * sub-chunks instead of once per sub-chunk (Algorithm 2). The path has four
+ * steps, exposed as three calls:
+ *
+ *   scale_build_reps      (a) block representative keys, sub-chunk
+ *                             fingerprints (Eq. 6) and anchor-based clusters
+ *                             (Eq. 8, Algorithm 1);
+ *   scale_select          (b) GQA-aware scoring of the representatives against
+ *                             each cluster's anchor fingerprint with head
+ *                             soft-voting, and (c) a deterministic top-k
+ *                             (Eq. 9, Sec. V-A3 "Selection function
+ *                             instantiation");
+ *   scale_sparse_prefill  (d) block-sparse causal attention over sinks,
+ *                             selected blocks and the cluster-spanning local
+ *                             window with an online softmax (Eq. 10).
+ *
+ * SCALE_MODE_PER_SUBCHUNK runs the same steps with every sub-chunk as its own
+ * unit: the per-sub-chunk (TokenSelect-style) baseline of Sec. III-A.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Layouts. Q and O: bf16 [N][H_q][d_h]; K and V: bf16 [N][H_kv][d_h]
+ *    (token-major, head_dim innermost, contiguous). Query head h reads KV head
+ *    h / (H_q / H_kv). Representatives: fp32 [H_kv][nb][d_h], nb = ceil(N/B).
+ *    Fingerprints: fp32 [M][H_q*d_h], M = ceil(N/L). Unit table: int32
+ *    unit_start[M+1], unit u covering sub-chunks [unit_start[u],
+ *    unit_start[u+1]), plus a device int32 n_units. Selection: int32
+ *    sel_blocks[M][top_k] (ascending, -1 padded) and int32 sel_count[M],
+ *    row u = unit u.
+ *  - Pointers. All data pointers are DEVICE pointers (except where a name says
+ *    _host), 16-byte aligned, owned by the caller. The library allocates no
+ *    memory on any path; scratch lives in a caller-provided workspace of
+ *    scale_workspace_size() bytes, initialised once with scale_workspace_init().
+ *  - Streams. `stream` is a cudaStream_t (NULL = legacy default stream). Calls
+ *    only enqueue work on it and never synchronise, except the functions
+ *    documented as synchronous (scale_get_device_status, scale_prefill_host).
+ *  - Errors. Argument problems are reported synchronously by the return value
+ *    (scale_status_t); nothing is enqueued then. Device-side problems (a
+ *    bounded wait that ran out, a failed bounds check) are recorded in a status
+ *    word inside the workspace and read with scale_get_device_status(). There
+ *    is no CPU fallback: every step runs in this library's CUDA kernels.
+ *  - Concurrency. Calls are reentrant; two calls that share a workspace must
+ *    not overlap on the GPU.
+ *  - Supported shapes: head_dim 128, H_q / H_kv even (for the attention call),
+ *    N < 2^31, outer_chunk a multiple of sub_chunk.
+ */
+#ifndef SCALE_H
+#define SCALE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A cudaStream_t; declared here so that the header needs no CUDA include. */
+typedef struct CUstream_st *scale_stream_t;
+
+typedef enum {
+    SCALE_OK = 0,
+    SCALE_ERR_INVALID_ARG = -1, /* a null/misaligned pointer or inconsistent sizes */
+    SCALE_ERR_UNSUPPORTED = -2, /* valid but outside what the kernels implement */
+    SCALE_ERR_WORKSPACE = -3,   /* workspace smaller than scale_workspace_size() */
+    SCALE_ERR_CUDA = -4,        /* a CUDA runtime call failed */
+    SCALE_ERR_TIMEOUT = -5,     /* device status: a bounded wait ran out */
+    SCALE_ERR_DEVICE = -6       /* device status: a device-side check failed */
+} scale_status_t;
+
+typedef enum {
+    SCALE_MODE_PER_CLUSTER = 0,  /* SCR: one selection per cluster (Algorithm 2) */
+    SCALE_MODE_PER_SUBCHUNK = 1  /* baseline: one selection per sub-chunk (Sec. III-A) */
+} scale_mode_t;
+
+/* Problem description. Notation of the paper in brackets. */
+typedef struct scale_params {
+    int32_t num_q_heads;           /* [H]  query heads                                   */
+    int32_t num_kv_heads;          /*      KV heads; divides num_q_heads (GQA)           */
+    int32_t head_dim;              /* [d_h] must be 128                                  */
+    int32_t sub_chunk;             /* [L]  sub-chunk length in tokens                    */
+    int64_t n_tokens;              /* [N]  tokens of Q, K and V                          */
+    int32_t max_cluster_subchunks; /* [L_max / L] cluster cap (Eq. 8)                    */
+    int32_t outer_chunk;           /* [L_outer] tokens; 0 means L_max; multiple of L     */
+    float theta;                   /* [theta] admission threshold (Eq. 8);
+                                      <= -1 admits every sub-chunk                       */
+    int32_t block_size;            /* [B]  KV block size of the selection, tokens        */
+    int32_t top_k;                 /* [k]  selected blocks per unit                      */
+    int32_t n_sink;                /* [n_init] leading sink tokens always attended       */
+    int32_t n_local;               /* [n_local^base] window before the unit's first token */
+    float select_scale;            /* sigma: logit scale inside the per-head softmax     */
+    float attn_scale;              /* softmax scale of Eq. 10; 0 means 1/sqrt(d_h)       */
+} scale_params_t;
+
+/* Bytes of workspace that scale_build_reps / scale_select / scale_sparse_prefill
+ * need for `p` and `mode` (one workspace serves all three). Synchronous, host only. */
+int scale_workspace_size(const scale_params_t *p, int32_t mode, size_t *bytes);
+
+/* Zero the workspace header (the device status word). Call once after
+ * allocating a workspace, and again to clear a recorded device error. */
+int scale_workspace_init(void *ws, size_t ws_bytes, scale_stream_t stream);
+
+/* Step (a). Eq. 6 and Sec. V-A1: fingerprints[i] = mean of the multi-head
+ * queries of sub-chunk i (tokens [iL, min(N,(i+1)L))); block representative
+ * key of block b and KV head j = mean of K over the tokens of the block;
+ * Algorithm 1 with the admission rule of Eq. 8 inside each outer chunk of
+ * outer_chunk tokens, producing unit_start[0..n_units] (entries after
+ * n_units are set to M) and *n_units (device).
+ *   q            bf16 [N][H_q][128]        k  bf16 [N][H_kv][128]
+ *   reps         fp32 [H_kv][nb][128]      out
+ *   fingerprints fp32 [M][H_q*128]         out (raw means v_i, not normalised)
+ *   unit_start   int32 [M+1]               out
+ *   n_units      int32 [1]                 out (device)
+ */
+int scale_build_reps(const scale_params_t *p, const void *q, const void *k, float *reps,
+                     float *fingerprints, int32_t *unit_start, int32_t *n_units, void *ws,
+                     size_t ws_bytes, scale_stream_t stream);
+
+/* Steps (b) and (c). Eq. 9 with head soft-voting (Sec. V-A3): for every unit u
+ * starting in [tok_begin, tok_end) (SCR: the clusters of unit_start; baseline:
+ * the sub-chunks) with anchor sub-chunk a (its first), and every query head h:
+ *   z_{h,b} = select_scale * v_a^(h) . r_b^(h / g)
+ * over the candidate blocks b that hold a token in [n_sink, W_u),
+ * W_u = max(0, s_u - n_local); p_h = softmax_b(z_h); score_b = sum_h p_{h,b};
+ * the top_k blocks by (score descending, block index ascending), written to
+ * sel_blocks[u] in ascending order, -1 padded; sel_count[u] = min(top_k,
+ * |candidates|). tok_begin and tok_end must be multiples of outer_chunk (SCR)
+ * or sub_chunk (baseline), or tok_end == N.
+ *   sel_scores  fp32 [M][nb] or NULL: score_b on the candidates, NaN elsewhere.
+ * unit_start / n_units are ignored in baseline mode (may be NULL). */
+int scale_select(const scale_params_t *p, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                 const float *reps, const float *fingerprints, const int32_t *unit_start,
+                 const int32_t *n_units, int32_t *sel_blocks, int32_t *sel_count,
+                 float *sel_scores, void *ws, size_t ws_bytes, scale_stream_t stream);
+
+/* Step (d). Eq. 10 for every query row p of every unit u starting in
+ * [tok_begin, tok_end) and every query head h:
+ *   keys K(p) = ([0, n_sink) U selected blocks of u U [W_u, e_u)) n [0, p],
+ *   taken as a set (each key once), with W_u = max(0, s_u - n_local);
+ *   out[p][h] = sum_{t in K(p)} softmax_t(attn_scale * q_p^(h) . k_t^(h/g)) v_t^(h/g)
+ * computed with bf16 tensor-core products, fp32 accumulation and an online
+ * softmax; probabilities are rounded to bf16 before the product with V; out
+ * is rounded to bf16 (nearest even). Rows outside [tok_begin, tok_end) are
+ * not written. Same range rule as scale_select.
+ *   q, out bf16 [N][H_q][128];  k, v bf16 [N][H_kv][128];
+ *   sel_blocks / sel_count as written by scale_select (any selection obeying
+ *   the same layout is accepted; entries outside [0, nb) are ignored). */
+int scale_sparse_prefill(const scale_params_t *p, int32_t mode, int64_t tok_begin,
+                         int64_t tok_end, const void *q, const void *k, const void *v,
+                         const int32_t *unit_start, const int32_t *n_units,
+                         const int32_t *sel_blocks, const int32_t *sel_count, void *out,
+                         void *ws, size_t ws_bytes, scale_stream_t stream);
+
+/* Synchronous: waits for `stream`, then reads the device status word of `ws`
+ * into *status (SCALE_OK, SCALE_ERR_TIMEOUT or SCALE_ERR_DEVICE). The word is
+ * sticky until scale_workspace_init(). */
+int scale_get_device_status(const void *ws, scale_stream_t stream, int32_t *status);
+
+/* Host-only bookkeeping of the cost model of Sec. V-A2: given a unit table in
+ * HOST memory, the number of units and how many of them make a retrieval call
+ * (non-empty candidate set). Baseline mode ignores unit_start_host. */
+int scale_retrieval_calls(const scale_params_t *p, int32_t mode, const int32_t *unit_start_host,
+                          int32_t n_units, int64_t *units, int64_t *calls);
+
+/* End to end from HOST buffers: copies q, k, v (host, bf16 layouts above) to
+ * the device, runs steps (a)-(d) over all tokens, copies the attention output
+ * back to out_host, and waits for `stream`. `arena` is a caller-owned device
+ * buffer of scale_prefill_host_arena_size() bytes that holds the device copies,
+ * the intermediate tensors and the workspace. Host buffers may be pageable;
+ * pinned buffers make the copies asynchronous with respect to the host. */
+int scale_prefill_host_arena_size(const scale_params_t *p, int32_t mode, size_t *bytes);
+int scale_prefill_host(const scale_params_t *p, int32_t mode, const void *q_host,
+                       const void *k_host, const void *v_host, void *out_host, void *arena,
+                       size_t arena_bytes, scale_stream_t stream);
+
+/* Upper bound, in nanoseconds of wall time, of every device-side wait of the
+ * attention kernel (default 4e9). A wait that runs out records
+ * SCALE_ERR_TIMEOUT in the device status and the kernel returns. Process-wide. */
+int scale_set_wait_timeout_ns(uint64_t ns);
+
+/* Self-check of the bounded-wait machinery: launches one block that waits on an
+ * mbarrier nothing arrives at, with a limit of `timeout_ns`; the kernel records
+ * SCALE_ERR_TIMEOUT in the device status of `ws` and returns. */
+int scale_selftest_wait_timeout(void *ws, size_t ws_bytes, uint64_t timeout_ns,
+                                scale_stream_t stream);
+
+const char *scale_status_string(int status);
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+int scale_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SCALE_H */

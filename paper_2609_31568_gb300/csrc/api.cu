@@ -1,0 +1,343 @@
+// api.cu -- the extern "C" boundary of libscale: argument validation, the
+// workspace layout, the launch of each step on the caller's stream, and the
+// end-to-end call that works from host buffers.
+#include <atomic>
+#include <cmath>
+
+#include "scale_internal.h"
+
+namespace scale {
+
+static std::atomic<uint64_t> g_timeout_ns{4000000000ull};
+
+int derive(const scale_params_t* p, Derived* d)
+{
+    if (!p || !d) return SCALE_ERR_INVALID_ARG;
+    if (p->num_q_heads <= 0 || p->num_kv_heads <= 0 || p->num_q_heads % p->num_kv_heads)
+        return SCALE_ERR_INVALID_ARG;
+    if (p->head_dim != kHeadDim) return SCALE_ERR_UNSUPPORTED;
+    if (p->n_tokens <= 0 || p->sub_chunk <= 0 || p->max_cluster_subchunks <= 0 ||
+        p->outer_chunk < 0 || p->block_size <= 0 || p->top_k < 0 || p->n_sink < 0 ||
+        p->n_local < 0)
+        return SCALE_ERR_INVALID_ARG;
+    if (std::isnan(p->theta) || !std::isfinite(p->select_scale) || !std::isfinite(p->attn_scale) ||
+        p->attn_scale < 0.f)
+        return SCALE_ERR_INVALID_ARG;
+    const int64_t L_outer = p->outer_chunk ? p->outer_chunk
+                                           : static_cast<int64_t>(p->max_cluster_subchunks) * p->sub_chunk;
+    if (L_outer % p->sub_chunk) return SCALE_ERR_INVALID_ARG;
+    const int g = p->num_q_heads / p->num_kv_heads;
+    if (g > 32 || p->num_kv_heads > 64) return SCALE_ERR_UNSUPPORTED;
+    if (p->n_tokens >= (1ll << 31) - 256) return SCALE_ERR_UNSUPPORTED;
+    d->N = p->n_tokens;
+    d->Hq = p->num_q_heads;
+    d->Hkv = p->num_kv_heads;
+    d->g = g;
+    d->dh = p->head_dim;
+    d->L = p->sub_chunk;
+    d->S_max = p->max_cluster_subchunks;
+    d->per_outer = static_cast<int>(L_outer / p->sub_chunk);
+    d->B = p->block_size;
+    d->k = p->top_k;
+    d->n_sink = p->n_sink;
+    d->n_local = p->n_local;
+    d->M = (d->N + d->L - 1) / d->L;
+    d->nb = (d->N + d->B - 1) / d->B;
+    d->D = d->Hq * kHeadDim;
+    d->fp_splits = (d->L + 511) / 512;
+    d->theta = p->theta;
+    d->sigma = p->select_scale;
+    d->attn_scale = p->attn_scale > 0.f ? p->attn_scale : 1.0f / std::sqrt(static_cast<float>(kHeadDim));
+    return SCALE_OK;
+}
+
+WsLayout ws_layout(const Derived& d)
+{
+    WsLayout w{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off = align_up(off + bytes, kAlign);
+        return at;
+    };
+    w.status = take(256);
+    w.fp_partial = take(static_cast<size_t>(d.M) * d.fp_splits * d.D * sizeof(float));
+    w.norms = take(static_cast<size_t>(d.M) * sizeof(float));
+    w.gram = take(static_cast<size_t>(d.M) * d.S_max * sizeof(float));
+    w.anchor = take(static_cast<size_t>(d.M) * sizeof(int32_t));
+    w.logits = take(static_cast<size_t>(d.M) * d.Hq * d.nb * sizeof(float));
+    w.stats = take(static_cast<size_t>(d.M) * d.Hq * 2 * sizeof(float));
+    w.scores = take(static_cast<size_t>(d.M) * d.nb * sizeof(float));
+    w.total = off;
+    return w;
+}
+
+namespace {
+
+bool aligned(const void* ptr, size_t a) { return (reinterpret_cast<uintptr_t>(ptr) % a) == 0; }
+
+// A device (or managed) allocation visible to the current device.
+bool device_ptr(const void* ptr, size_t align)
+{
+    if (!ptr || !aligned(ptr, align)) return false;
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+int check_ws(const Derived& d, const void* ws, size_t ws_bytes)
+{
+    if (!device_ptr(ws, 256)) return SCALE_ERR_INVALID_ARG;
+    if (ws_bytes < ws_layout(d).total) return SCALE_ERR_WORKSPACE;
+    return SCALE_OK;
+}
+
+int check_range(const Derived& d, int mode, int64_t tb, int64_t te)
+{
+    if (mode != SCALE_MODE_PER_CLUSTER && mode != SCALE_MODE_PER_SUBCHUNK) return SCALE_ERR_INVALID_ARG;
+    if (tb < 0 || te < tb || te > d.N) return SCALE_ERR_INVALID_ARG;
+    const int64_t unit = mode == SCALE_MODE_PER_CLUSTER ? static_cast<int64_t>(d.per_outer) * d.L : d.L;
+    if (tb % unit) return SCALE_ERR_INVALID_ARG;
+    if (te != d.N && te % unit) return SCALE_ERR_INVALID_ARG;
+    return SCALE_OK;
+}
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? SCALE_OK : SCALE_ERR_CUDA; }
+
+struct Arena {
+    size_t q, k, v, out, reps, fp, unit_start, n_units, sel, sel_count, ws, total;
+};
+
+Arena arena_layout(const Derived& d, int mode)
+{
+    (void)mode;
+    Arena a{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off = align_up(off + bytes, kAlign);
+        return at;
+    };
+    a.q = take(static_cast<size_t>(d.N) * d.Hq * kHeadDim * 2);
+    a.k = take(static_cast<size_t>(d.N) * d.Hkv * kHeadDim * 2);
+    a.v = take(static_cast<size_t>(d.N) * d.Hkv * kHeadDim * 2);
+    a.out = take(static_cast<size_t>(d.N) * d.Hq * kHeadDim * 2);
+    a.reps = take(static_cast<size_t>(d.Hkv) * d.nb * kHeadDim * sizeof(float));
+    a.fp = take(static_cast<size_t>(d.M) * d.D * sizeof(float));
+    a.unit_start = take(static_cast<size_t>(d.M + 1) * sizeof(int32_t));
+    a.n_units = take(sizeof(int32_t));
+    a.sel = take(static_cast<size_t>(d.M) * (d.k > 0 ? d.k : 1) * sizeof(int32_t));
+    a.sel_count = take(static_cast<size_t>(d.M) * sizeof(int32_t));
+    a.ws = take(ws_layout(d).total);
+    a.total = off;
+    return a;
+}
+
+}  // namespace
+}  // namespace scale
+
+using namespace scale;
+
+extern "C" {
+
+int scale_version(void) { return 10000; }
+
+const char* scale_status_string(int s)
+{
+    switch (s) {
+    case SCALE_OK: return "ok";
+    case SCALE_ERR_INVALID_ARG: return "invalid argument";
+    case SCALE_ERR_UNSUPPORTED: return "unsupported parameters";
+    case SCALE_ERR_WORKSPACE: return "workspace too small";
+    case SCALE_ERR_CUDA: return "CUDA runtime error";
+    case SCALE_ERR_TIMEOUT: return "device wait timed out";
+    case SCALE_ERR_DEVICE: return "device-side check failed";
+    default: return "unknown status";
+    }
+}
+
+int scale_workspace_size(const scale_params_t* p, int32_t mode, size_t* bytes)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (!bytes || (mode != SCALE_MODE_PER_CLUSTER && mode != SCALE_MODE_PER_SUBCHUNK))
+        return SCALE_ERR_INVALID_ARG;
+    *bytes = ws_layout(d).total;
+    return SCALE_OK;
+}
+
+int scale_workspace_init(void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    if (!device_ptr(ws, 256) || ws_bytes < 256) return SCALE_ERR_INVALID_ARG;
+    return cuda_status(cudaMemsetAsync(ws, 0, 256, stream));
+}
+
+int scale_build_reps(const scale_params_t* p, const void* q, const void* k, float* reps,
+                     float* fingerprints, int32_t* unit_start, int32_t* n_units, void* ws,
+                     size_t ws_bytes, scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(reps, 16) ||
+        !device_ptr(fingerprints, 16) || !device_ptr(unit_start, 4) || !device_ptr(n_units, 4))
+        return SCALE_ERR_INVALID_ARG;
+    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
+    return cuda_status(launch_build_reps(d, q, k, reps, fingerprints, unit_start, n_units,
+                                         static_cast<uint8_t*>(ws), stream));
+}
+
+int scale_select(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                 const float* reps, const float* fingerprints, const int32_t* unit_start,
+                 const int32_t* n_units, int32_t* sel_blocks, int32_t* sel_count,
+                 float* sel_scores, void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
+    if (!device_ptr(reps, 16) || !device_ptr(fingerprints, 16) || !device_ptr(sel_count, 4) ||
+        (d.k > 0 && !device_ptr(sel_blocks, 4)) || (sel_scores && !device_ptr(sel_scores, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if (mode == SCALE_MODE_PER_CLUSTER && (!device_ptr(unit_start, 4) || !device_ptr(n_units, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
+    if (tok_begin == tok_end) return SCALE_OK;
+    return cuda_status(launch_select(d, mode, tok_begin, tok_end, reps, fingerprints, unit_start,
+                                     n_units, sel_blocks, sel_count, sel_scores,
+                                     static_cast<uint8_t*>(ws), stream));
+}
+
+int scale_sparse_prefill(const scale_params_t* p, int32_t mode, int64_t tok_begin,
+                         int64_t tok_end, const void* q, const void* k, const void* v,
+                         const int32_t* unit_start, const int32_t* n_units,
+                         const int32_t* sel_blocks, const int32_t* sel_count, void* out,
+                         void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
+    if (d.g % 2) return SCALE_ERR_UNSUPPORTED;
+    if (max_distant_segments(d) > kMaxSegments) return SCALE_ERR_UNSUPPORTED;
+    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(v, 16) || !device_ptr(out, 16) ||
+        !device_ptr(sel_count, 4) || (d.k > 0 && !device_ptr(sel_blocks, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if (mode == SCALE_MODE_PER_CLUSTER && (!device_ptr(unit_start, 4) || !device_ptr(n_units, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
+    if (tok_begin == tok_end) return SCALE_OK;
+    return cuda_status(launch_sparse_prefill(d, mode, tok_begin, tok_end, q, k, v, unit_start,
+                                             n_units, sel_blocks, sel_count, out,
+                                             static_cast<uint8_t*>(ws), g_timeout_ns.load(),
+                                             stream));
+}
+
+int scale_get_device_status(const void* ws, scale_stream_t stream, int32_t* status)
+{
+    if (!device_ptr(ws, 256) || !status) return SCALE_ERR_INVALID_ARG;
+    int32_t h = 0;
+    cudaError_t e = cudaMemcpyAsync(&h, static_cast<const uint8_t*>(ws) + kStatusOffset, sizeof h,
+                                    cudaMemcpyDeviceToHost, stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return SCALE_ERR_CUDA;
+    *status = h;
+    return SCALE_OK;
+}
+
+int scale_retrieval_calls(const scale_params_t* p, int32_t mode, const int32_t* unit_start_host,
+                          int32_t n_units, int64_t* units, int64_t* calls)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (!units || !calls || (mode != SCALE_MODE_PER_CLUSTER && mode != SCALE_MODE_PER_SUBCHUNK))
+        return SCALE_ERR_INVALID_ARG;
+    const bool per_sub = mode == SCALE_MODE_PER_SUBCHUNK;
+    if (!per_sub && (!unit_start_host || n_units < 0 || n_units > d.M)) return SCALE_ERR_INVALID_ARG;
+    const int64_t n = per_sub ? d.M : n_units;
+    int64_t c = 0;
+    for (int64_t u = 0; u < n; ++u) {
+        const int64_t a = per_sub ? u : unit_start_host[u];
+        if (a < 0 || a >= d.M) return SCALE_ERR_INVALID_ARG;
+        const int64_t s = a * d.L;
+        const int64_t W = s - d.n_local > 0 ? s - d.n_local : 0;
+        const int64_t lo = d.n_sink / d.B;
+        int64_t hi = (W + d.B - 1) / d.B;
+        if (hi > d.nb) hi = d.nb;
+        if (hi > lo) ++c;
+    }
+    *units = n;
+    *calls = c;
+    return SCALE_OK;
+}
+
+int scale_prefill_host_arena_size(const scale_params_t* p, int32_t mode, size_t* bytes)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (!bytes || (mode != SCALE_MODE_PER_CLUSTER && mode != SCALE_MODE_PER_SUBCHUNK))
+        return SCALE_ERR_INVALID_ARG;
+    *bytes = arena_layout(d, mode).total;
+    return SCALE_OK;
+}
+
+int scale_prefill_host(const scale_params_t* p, int32_t mode, const void* q_host,
+                       const void* k_host, const void* v_host, void* out_host, void* arena,
+                       size_t arena_bytes, scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (mode != SCALE_MODE_PER_CLUSTER && mode != SCALE_MODE_PER_SUBCHUNK) return SCALE_ERR_INVALID_ARG;
+    if (!q_host || !k_host || !v_host || !out_host || !device_ptr(arena, 256))
+        return SCALE_ERR_INVALID_ARG;
+    const Arena A = arena_layout(d, mode);
+    if (arena_bytes < A.total) return SCALE_ERR_WORKSPACE;
+    uint8_t* base = static_cast<uint8_t*>(arena);
+    const size_t qb = static_cast<size_t>(d.N) * d.Hq * kHeadDim * 2;
+    const size_t kb = static_cast<size_t>(d.N) * d.Hkv * kHeadDim * 2;
+    cudaError_t e = cudaMemcpyAsync(base + A.q, q_host, qb, cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(base + A.k, k_host, kb, cudaMemcpyHostToDevice, stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(base + A.v, v_host, kb, cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return SCALE_ERR_CUDA;
+    void* ws = base + A.ws;
+    const size_t wsb = arena_bytes - A.ws;
+    auto* reps = reinterpret_cast<float*>(base + A.reps);
+    auto* fp = reinterpret_cast<float*>(base + A.fp);
+    auto* us = reinterpret_cast<int32_t*>(base + A.unit_start);
+    auto* nu = reinterpret_cast<int32_t*>(base + A.n_units);
+    auto* sel = reinterpret_cast<int32_t*>(base + A.sel);
+    auto* cnt = reinterpret_cast<int32_t*>(base + A.sel_count);
+    if ((rc = scale_workspace_init(ws, wsb, stream))) return rc;
+    if ((rc = scale_build_reps(p, base + A.q, base + A.k, reps, fp, us, nu, ws, wsb, stream))) return rc;
+    if ((rc = scale_select(p, mode, 0, d.N, reps, fp, us, nu, sel, cnt, nullptr, ws, wsb, stream))) return rc;
+    if ((rc = scale_sparse_prefill(p, mode, 0, d.N, base + A.q, base + A.k, base + A.v, us, nu, sel,
+                                   cnt, base + A.out, ws, wsb, stream)))
+        return rc;
+    e = cudaMemcpyAsync(out_host, base + A.out, qb, cudaMemcpyDeviceToHost, stream);
+    if (e != cudaSuccess) return SCALE_ERR_CUDA;
+    int32_t st = 0;
+    if ((rc = scale_get_device_status(ws, stream, &st))) return rc;
+    return st;
+}
+
+int scale_set_wait_timeout_ns(uint64_t ns)
+{
+    if (ns == 0) return SCALE_ERR_INVALID_ARG;
+    g_timeout_ns.store(ns);
+    return SCALE_OK;
+}
+
+int scale_selftest_wait_timeout(void* ws, size_t ws_bytes, uint64_t timeout_ns, scale_stream_t stream)
+{
+    if (!device_ptr(ws, 256) || ws_bytes < 256 || timeout_ns == 0) return SCALE_ERR_INVALID_ARG;
+    return cuda_status(launch_wait_selftest(static_cast<uint8_t*>(ws), timeout_ns, stream));
+}
+
+}  // extern "C"

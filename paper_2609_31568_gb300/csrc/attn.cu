@@ -1,0 +1,500 @@
+// attn.cu -- step (d) of the SCR prefill path: block-sparse causal attention
+// over the cluster (Eq. 10, Sec. V-A3 "Sparse attention over the cluster").
+//
+// For a query row p of unit u = [s_u, e_u) the key set is
+//   K(p) = D_u  U  [W_u, p],   D_u = ([0, n_sink) U selected blocks) n [0, W_u),
+// W_u = max(0, s_u - n_local): the distant part D_u is shared by every row of
+// the unit (the anchor-shared retrieval), the local part is the cluster-
+// spanning window with the causal mask. Because D_u lies below W_u and the
+// window starts at W_u, the two never overlap, and D_u is built from the sink
+// range and each selected block clipped to [n_sink, W_u), so every key is
+// visited once (the de-duplication of Sec. V-A3).
+//
+// Design (one CTA per work item = 128 query rows x 2 query heads of one KV head):
+//  - D_u is cut into 64-row segments; two segments form a 128-key tile. Each
+//    segment is one TMA box per 64-column half of head_dim, so gathered blocks
+//    land in shared memory in the 128-byte-swizzled K-major layout the tensor
+//    cores read, with no copy through registers.
+//  - warp 8 (one thread) issues TMA loads: both Q tiles once, then K and V
+//    tiles into a 2-stage ring;
+//  - warp 9 (one thread) issues tcgen05.mma: S_q = Q_q K^T into TMEM, and
+//    O_q += P_q V with P read from TMEM (bf16, written over S_q);
+//  - warps 0-3 and 4-7 run the online softmax of Q tile 0 and 1, one thread
+//    per row (= TMEM lane), and the epilogue. The running max is raised only
+//    when it grows by more than 8 (log2 units), so O is rescaled rarely; the
+//    final normalisation uses the same max, which keeps the result exact.
+//  - Every wait is bounded in wall time; on expiry the kernel records
+//    SCALE_ERR_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and
+//    returns.
+#include <cuda_bf16.h>
+
+#include "ptx_sm103.cuh"
+#include "scale_internal.h"
+#include "tma_host.h"
+
+namespace scale {
+namespace {
+
+using namespace scale_ptx;
+
+constexpr int kThreads = 320;
+constexpr int kRows = 128;                    // query rows per Q tile
+constexpr uint32_t kTileBytes = 128 * 128 * 2;  // one 128 x 128 bf16 tile
+constexpr uint32_t kHalf = kTileBytes / 2;    // one 64-column half (128 rows x 128 B)
+constexpr uint32_t kSegBytes = 64 * 128;      // one 64-row x 64-column box
+constexpr float kRescaleThreshold = 8.0f;     // log2 units
+
+// Dynamic shared memory map (offsets from the 1024-aligned base).
+constexpr uint32_t kOffQ = 0;                          // 2 Q tiles
+constexpr uint32_t kOffK = kOffQ + 2 * kTileBytes;     // 2 K stages
+constexpr uint32_t kOffV = kOffK + 2 * kTileBytes;     // 2 V stages
+constexpr uint32_t kOffSeg = kOffV + 2 * kTileBytes;   // int2 segment table
+constexpr uint32_t kSmemBytes = kOffSeg + kMaxSegments * 8 + 1024;
+
+struct AttnArgs {
+    Units ut;
+    int sc_begin, sc_end;
+    int units_max;  // grid extent over units
+    int qb_max;     // grid extent over 128-row query blocks of one unit
+    int Hq, Hkv, g, pairs;
+    int64_t N, nb;
+    int B, k, n_sink, n_local;
+    float scale_log2;
+    const int32_t* sel;
+    const int32_t* sel_count;
+    __nv_bfloat16* out;
+    int32_t* status;
+    uint64_t timeout_ns;
+};
+
+struct Barriers {
+    uint64_t q_full;
+    uint64_t k_full[2], v_full[2], k_empty[2], v_empty[2];
+    uint64_t s_full[2];  // S of Q tile q ready (and every earlier MMA of the CTA done)
+    uint64_t p_full[2];  // P of Q tile q written (128 arrivals)
+    uint64_t o_full;     // last P.V of both tiles done
+    uint64_t drain;
+};
+
+__device__ __forceinline__ void fail(volatile int* abort_flag, int32_t* status)
+{
+    *abort_flag = 1;
+    record_status(status, SCALE_ERR_TIMEOUT);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
+              const __grid_constant__ CUtensorMap tv, const AttnArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ Barriers bars;
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+    __shared__ int s_nseg;
+
+    // ---- work item: heaviest (last) query blocks first ----
+    int lin = blockIdx.x;
+    const int hp = lin % (a.Hkv * a.pairs);
+    lin /= a.Hkv * a.pairs;
+    const int ul = lin % a.units_max;
+    const int qb = a.qb_max - 1 - lin / a.units_max;
+    const int kvh = hp / a.pairs;
+    const int h0 = kvh * a.g + 2 * (hp % a.pairs);
+
+    const int u = unit_lower_bound(a.ut, a.sc_begin) + ul;
+    if (u >= unit_lower_bound(a.ut, a.sc_end)) return;
+    int anchor;
+    int64_t s_u, e_u;
+    unit_range(a.ut, u, &anchor, &s_u, &e_u);
+    const int64_t q0 = s_u + static_cast<int64_t>(kRows) * qb;
+    if (q0 >= e_u) return;
+    const int64_t q_end = (q0 + kRows < e_u) ? q0 + kRows : e_u;
+    const int64_t W = (s_u - a.n_local > 0) ? s_u - a.n_local : 0;
+    const int n_lt = static_cast<int>((q_end - W + 127) / 128);
+
+    uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+    int2* seg = reinterpret_cast<int2*>(smem + kOffSeg);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    if (tid == 0) {
+        abort_flag = 0;
+        mbar_init(&bars.q_full, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&bars.k_full[i], 1);
+            mbar_init(&bars.v_full[i], 1);
+            mbar_init(&bars.k_empty[i], 1);
+            mbar_init(&bars.v_empty[i], 1);
+            mbar_init(&bars.s_full[i], 1);
+            mbar_init(&bars.p_full[i], 128);
+        }
+        mbar_init(&bars.o_full, 1);
+        mbar_init(&bars.drain, 1);
+        fence_barrier_init();
+    }
+    if (warp == 9) {
+        tmem_alloc(&tmem_slot, 512);
+        tmem_relinquish();
+    }
+    if (warp == 8) {
+        // Distant segments: the sinks, then each selected block clipped to
+        // [n_sink, W); 64 rows at most per segment.
+        const int64_t sink_end = a.n_sink < W ? a.n_sink : W;
+        const int n_sink_seg = static_cast<int>((sink_end + 63) / 64);
+        for (int i = lane; i < n_sink_seg; i += 32) {
+            const int64_t t0 = 64ll * i;
+            seg[i] = make_int2(static_cast<int>(t0), static_cast<int>(sink_end - t0 < 64 ? sink_end - t0 : 64));
+        }
+        int base = n_sink_seg;
+        int cnt = a.sel_count[u];
+        cnt = cnt < 0 ? 0 : (cnt > a.k ? a.k : cnt);
+        const int32_t* sl = a.sel + static_cast<int64_t>(u) * a.k;
+        bool overflow = false;
+        for (int c0 = 0; c0 < cnt; c0 += 32) {
+            const int i = c0 + lane;
+            int nseg = 0;
+            int64_t lo = 0, hi = 0;
+            if (i < cnt) {
+                const int64_t b = sl[i];
+                const int64_t prev = i > 0 ? sl[i - 1] : -1;
+                if (b >= 0 && b < a.nb && b > prev) {
+                    lo = b * a.B > a.n_sink ? b * a.B : a.n_sink;
+                    hi = (b + 1) * a.B < W ? (b + 1) * a.B : W;
+                    if (hi > lo) nseg = static_cast<int>((hi - lo + 63) / 64);
+                }
+            }
+            int incl = nseg;
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+                if (lane >= o) incl += y;
+            }
+            const int off = base + incl - nseg;
+            if (off + nseg > kMaxSegments - 1) overflow = true;
+            else
+                for (int m = 0; m < nseg; ++m) {
+                    const int64_t t0 = lo + 64ll * m;
+                    seg[off + m] = make_int2(static_cast<int>(t0), static_cast<int>(hi - t0 < 64 ? hi - t0 : 64));
+                }
+            base += __shfl_sync(0xFFFFFFFFu, incl, 31);
+        }
+        overflow = __any_sync(0xFFFFFFFFu, overflow);
+        if (lane == 0) {
+            if (overflow) {
+                record_status(a.status, SCALE_ERR_DEVICE);
+                base = 0;
+            }
+            if (base & 1) seg[base] = make_int2(0, 0);
+            s_nseg = base;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    const int n_dt = (s_nseg + 1) / 2;
+    const int T = n_dt + n_lt;
+
+    if (warp == 8) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tq);
+            tma_prefetch_desc(&tk);
+            tma_prefetch_desc(&tv);
+            mbar_arrive_expect_tx(&bars.q_full, 2 * kTileBytes);
+            for (int qt = 0; qt < 2; ++qt)
+                for (int hf = 0; hf < 2; ++hf)
+                    tma_load_3d(smem + kOffQ + qt * kTileBytes + hf * kHalf, &tq, &bars.q_full,
+                                hf * 64, h0 + qt, static_cast<int32_t>(q0));
+            int issued_k0 = 0, issued_k1 = 0, issued_v0 = 0, issued_v1 = 0;
+            for (int t = 0; t < T && !abort_flag; ++t) {
+                const int st = t & 1;
+                const uint32_t ph = ((t >> 1) - 1) & 1;
+                int32_t ta, tb;
+                if (t < n_dt) {
+                    ta = seg[2 * t].x;
+                    tb = seg[2 * t + 1].x;
+                } else {
+                    ta = static_cast<int32_t>(W + 128ll * (t - n_dt));
+                    tb = ta + 64;
+                }
+                if (t >= 2 && !mbar_wait_bounded(&bars.k_empty[st], ph, a.timeout_ns, &abort_flag)) {
+                    fail(&abort_flag, a.status);
+                    break;
+                }
+                mbar_arrive_expect_tx(&bars.k_full[st], kTileBytes);
+                if (st) ++issued_k1; else ++issued_k0;
+                uint8_t* kd = smem + kOffK + st * kTileBytes;
+                for (int hf = 0; hf < 2; ++hf) {
+                    tma_load_3d(kd + hf * kHalf, &tk, &bars.k_full[st], hf * 64, kvh, ta);
+                    tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.k_full[st], hf * 64, kvh, tb);
+                }
+                if (t >= 2 && !mbar_wait_bounded(&bars.v_empty[st], ph, a.timeout_ns, &abort_flag)) {
+                    fail(&abort_flag, a.status);
+                    break;
+                }
+                mbar_arrive_expect_tx(&bars.v_full[st], kTileBytes);
+                if (st) ++issued_v1; else ++issued_v0;
+                uint8_t* vd = smem + kOffV + st * kTileBytes;
+                for (int hf = 0; hf < 2; ++hf) {
+                    tma_load_3d(vd + hf * kHalf, &tv, &bars.v_full[st], hf * 64, kvh, ta);
+                    tma_load_3d(vd + hf * kHalf + kSegBytes, &tv, &bars.v_full[st], hf * 64, kvh, tb);
+                }
+            }
+            if (abort_flag) {
+                // Drain: wait (bounded, ignoring the abort flag) for the last
+                // phase of every buffer that received copies.
+                mbar_wait_bounded(&bars.q_full, 0, a.timeout_ns, nullptr);
+                if (issued_k0) mbar_wait_bounded(&bars.k_full[0], (issued_k0 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_k1) mbar_wait_bounded(&bars.k_full[1], (issued_k1 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_v0) mbar_wait_bounded(&bars.v_full[0], (issued_v0 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_v1) mbar_wait_bounded(&bars.v_full[1], (issued_v1 - 1) & 1, a.timeout_ns, nullptr);
+            }
+        }
+    } else if (warp == 9) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t id_qk = idesc_bf16_f32(128, 128, 0);
+            const uint32_t id_pv = idesc_bf16_f32(128, 128, 1);
+            const uint32_t q_base = smem_addr(smem + kOffQ);
+            const uint32_t k_base = smem_addr(smem + kOffK);
+            const uint32_t v_base = smem_addr(smem + kOffV);
+            bool ok = mbar_wait_bounded(&bars.q_full, 0, a.timeout_ns, &abort_flag);
+            auto issue_pv = [&](int t, int qt) {
+                const uint32_t vs = v_base + (t & 1) * kTileBytes;
+                const uint32_t d = tmem + qt * 256 + 128;
+                const uint32_t p = tmem + qt * 256;
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk)
+                    mma_ts(d, p + kk * 8, sdesc_sw128(vs + kk * 2048, kHalf, 1024), id_pv, (t > 0 || kk > 0) ? 1u : 0u);
+            };
+            for (int t = 0; ok && t < T; ++t) {
+                const int st = t & 1;
+                if (!mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t ks = k_base + st * kTileBytes;
+                for (int qt = 0; qt < 2; ++qt) {
+                    if (t > 0) {
+                        if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                        if (qt == 0 && !mbar_wait_bounded(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                        tc_fence_after();
+                        issue_pv(t - 1, qt);
+                    }
+                    const uint32_t qs = q_base + qt * kTileBytes;
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
+                        mma_ss(tmem + qt * 256, sdesc_sw128(qs + off, 16, 1024), sdesc_sw128(ks + off, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(&bars.s_full[qt]);
+                }
+                if (!ok) break;
+                mma_commit(&bars.k_empty[st]);
+                if (t > 0) mma_commit(&bars.v_empty[(t - 1) & 1]);
+            }
+            if (ok) {
+                for (int qt = 0; qt < 2 && ok; ++qt) {
+                    if (!mbar_wait_bounded(&bars.p_full[qt], (T - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                    if (qt == 0 && !mbar_wait_bounded(&bars.v_full[(T - 1) & 1], ((T - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                    tc_fence_after();
+                    issue_pv(T - 1, qt);
+                }
+                if (ok) mma_commit(&bars.o_full);
+            }
+            if (!ok) {
+                fail(&abort_flag, a.status);
+                // Drain: every MMA issued so far completes before TMEM is freed.
+                mma_commit(&bars.drain);
+                mbar_wait_bounded(&bars.drain, 0, a.timeout_ns, nullptr);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ softmax + epilogue
+        const int qt = warp >> 2;
+        const int quarter = warp & 3;
+        const int r = quarter * 32 + lane;
+        const int64_t p = q0 + r;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        const uint32_t s_addr = lane_base + qt * 256;
+        const uint32_t o_addr = s_addr + 128;
+        float m_run = -INFINITY, l_run = 0.f;
+        float s[128];
+        bool ok = true;
+        for (int t = 0; t < T; ++t) {
+            // tcgen05.ld/st are warp-collective: the outcome must be warp-uniform.
+            const bool got = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.s_full[qt], t & 1, a.timeout_ns, &abort_flag));
+            if (!got) { ok = false; break; }
+            tc_fence_after();
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t v[32];
+                tmem_ld32(s_addr + c * 32, v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(v[i]);
+            }
+            if (t < n_dt) {
+                const int la = seg[2 * t].y, lb = seg[2 * t + 1].y;
+                if (la < 64 || lb < 64) {
+#pragma unroll
+                    for (int c = 0; c < 128; ++c)
+                        if ((c < 64 ? c : c - 64) >= (c < 64 ? la : lb)) s[c] = -INFINITY;
+                }
+            } else {
+                const int64_t kb = W + 128ll * (t - n_dt);
+                if (kb + 127 > q0) {
+                    const int64_t lim = p - kb;  // keys kb + c with c > lim are in the future
+#pragma unroll
+                    for (int c = 0; c < 128; ++c)
+                        if (c > lim) s[c] = -INFINITY;
+                }
+            }
+            float mx = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 128; ++c) mx = fmaxf(mx, s[c]);
+            const float m_new = fmaxf(m_run, mx * a.scale_log2);
+            if (m_new > m_run + kRescaleThreshold) {
+                const float alpha = ex2(m_run - m_new);
+                l_run *= alpha;
+                if (t > 0) {
+#pragma unroll 1
+                    for (int c = 0; c < 8; ++c) {
+                        uint32_t v[16];
+                        tmem_ld16(o_addr + c * 16, v);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+                        tmem_st16(o_addr + c * 16, v);
+                    }
+                }
+                m_run = m_new;
+            }
+            const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
+            float sum = 0.f;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                uint32_t pk[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const float p0 = ex2(fmaf(s[h * 64 + 2 * i], a.scale_log2, neg_m));
+                    const float p1 = ex2(fmaf(s[h * 64 + 2 * i + 1], a.scale_log2, neg_m));
+                    sum += p0 + p1;
+                    pk[i] = pack_bf16x2(p0, p1);
+                }
+                tmem_st32(s_addr + h * 32, pk);
+            }
+            l_run += sum;
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(&bars.p_full[qt]);
+        }
+        bool go = __all_sync(0xFFFFFFFFu, ok && !abort_flag);
+        if (go) go = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.o_full, 0, a.timeout_ns, &abort_flag));
+        if (go) {
+            tc_fence_after();
+            const float inv_l = l_run > 0.f ? 1.0f / l_run : 0.f;
+            const bool store = p < q_end;
+            uint4* dst = reinterpret_cast<uint4*>(a.out + (p * a.Hq + h0 + qt) * static_cast<int64_t>(kHeadDim));
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t v[32];
+                tmem_ld32(o_addr + c * 32, v);
+                tmem_ld_wait();
+                if (store) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        dst[c * 4 + i] = make_uint4(
+                            pack_bf16x2(__uint_as_float(v[8 * i + 0]) * inv_l, __uint_as_float(v[8 * i + 1]) * inv_l),
+                            pack_bf16x2(__uint_as_float(v[8 * i + 2]) * inv_l, __uint_as_float(v[8 * i + 3]) * inv_l),
+                            pack_bf16x2(__uint_as_float(v[8 * i + 4]) * inv_l, __uint_as_float(v[8 * i + 5]) * inv_l),
+                            pack_bf16x2(__uint_as_float(v[8 * i + 6]) * inv_l, __uint_as_float(v[8 * i + 7]) * inv_l));
+                }
+            }
+        } else {
+            fail(&abort_flag, a.status);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+// Bounded-wait self-check: wait on a barrier nothing arrives at.
+__global__ void k_wait_selftest(int32_t* status, uint64_t timeout_ns)
+{
+    __shared__ uint64_t bar;
+    __shared__ volatile int never;
+    if (threadIdx.x == 0) {
+        never = 0;
+        mbar_init(&bar, 1);
+        fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !mbar_wait_bounded(&bar, 0, timeout_ns, &never))
+        record_status(status, SCALE_ERR_TIMEOUT);
+}
+
+}  // namespace
+
+int64_t max_distant_segments(const Derived& d)
+{
+    // ceil(n_sink / 64) sink segments, at most ceil(B / 64) per selected block,
+    // plus one pad segment.
+    return (d.n_sink + 63) / 64 + static_cast<int64_t>(d.k) * ((d.B + 63) / 64) + 1;
+}
+
+cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
+                                  const void* q, const void* k, const void* v,
+                                  const int32_t* unit_start, const int32_t* n_units,
+                                  const int32_t* sel_blocks, const int32_t* sel_count, void* out,
+                                  uint8_t* ws, uint64_t timeout_ns, cudaStream_t st)
+{
+    CUtensorMap tq, tk, tv;
+    if (!scale_host::make_token_major_map(&tq, q, kHeadDim, d.Hq, d.N, 64, 128) ||
+        !scale_host::make_token_major_map(&tk, k, kHeadDim, d.Hkv, d.N, 64, 64) ||
+        !scale_host::make_token_major_map(&tv, v, kHeadDim, d.Hkv, d.N, 64, 64))
+        return cudaErrorInvalidValue;
+
+    AttnArgs a;
+    a.ut = Units{unit_start, n_units, mode == SCALE_MODE_PER_SUBCHUNK, d.N, d.L, static_cast<int>(d.M)};
+    a.sc_begin = static_cast<int>(tok_begin / d.L);
+    a.sc_end = static_cast<int>((tok_end + d.L - 1) / d.L);
+    a.units_max = a.sc_end - a.sc_begin;
+    if (a.units_max <= 0) return cudaSuccess;
+    const int64_t unit_tokens = static_cast<int64_t>(mode == SCALE_MODE_PER_SUBCHUNK ? 1 : d.S_max) * d.L;
+    a.qb_max = static_cast<int>((unit_tokens + kRows - 1) / kRows);
+    a.Hq = d.Hq;
+    a.Hkv = d.Hkv;
+    a.g = d.g;
+    a.pairs = d.g / 2;
+    a.N = d.N;
+    a.nb = d.nb;
+    a.B = d.B;
+    a.k = d.k;
+    a.n_sink = d.n_sink;
+    a.n_local = d.n_local;
+    a.scale_log2 = d.attn_scale * 1.4426950408889634f;
+    a.sel = sel_blocks;
+    a.sel_count = sel_count;
+    a.out = static_cast<__nv_bfloat16*>(out);
+    a.status = reinterpret_cast<int32_t*>(ws + kStatusOffset);
+    a.timeout_ns = timeout_ns;
+
+    cudaError_t e = cudaFuncSetAttribute(k_sparse_attn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kSmemBytes));
+    if (e != cudaSuccess) return e;
+    const int64_t grid = static_cast<int64_t>(a.units_max) * a.qb_max * d.Hkv * a.pairs;
+    if (grid <= 0 || grid > 0x7FFFFFFFll) return cudaErrorInvalidConfiguration;
+    k_sparse_attn<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tq, tk, tv, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(uint8_t* ws, uint64_t timeout_ns, cudaStream_t st)
+{
+    k_wait_selftest<<<1, 32, 0, st>>>(reinterpret_cast<int32_t*>(ws + kStatusOffset), timeout_ns);
+    return cudaGetLastError();
+}
+
+}  // namespace scale

@@ -1,0 +1,263 @@
+// reps.cu -- step (a) of the SCR prefill path: block representative keys,
+// sub-chunk fingerprints (Eq. 6) with their norms (Sec. V-A1), and
+// anchor-based clustering (Eq. 8, Algorithm 1) inside each outer chunk.
+//
+// All four kernels stream their inputs once from HBM with 16-byte loads and
+// reduce in a fixed order, so their results are bit-reproducible run to run.
+#include <cuda_bf16.h>
+
+#include "scale_internal.h"
+
+namespace scale {
+namespace {
+
+__device__ __forceinline__ void add_bf16x8(float (&acc)[8], const uint4 x)
+{
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        acc[2 * i] += __uint_as_float(w[i] << 16);
+        acc[2 * i + 1] += __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+}
+
+__device__ __forceinline__ uint4 ld_stream(const uint4* p)
+{
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+    return r;
+}
+
+// Representative key of block b for every KV head: the mean of the block's
+// keys. One CTA per block; thread c owns elements [8c, 8c+8) of the token row
+// (H_kv * 128 elements), so every token row is read as one coalesced span.
+__global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k, int64_t N,
+                                                      int row_chunks, int B, int64_t nb,
+                                                      float* __restrict__ reps)
+{
+    const int c = threadIdx.x;
+    if (c >= row_chunks) return;
+    const int64_t b = blockIdx.x;
+    const int64_t t0 = b * B;
+    const int64_t t1 = (t0 + B < N) ? t0 + B : N;
+    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    const uint4* src = k + t0 * row_chunks + c;
+    int64_t t = t0;
+    for (; t + 8 <= t1; t += 8) {
+        uint4 x[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = ld_stream(src + (t - t0 + i) * row_chunks);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) add_bf16x8(acc, x[i]);
+    }
+    for (; t < t1; ++t) add_bf16x8(acc, ld_stream(src + (t - t0) * row_chunks));
+    const float cnt = static_cast<float>(t1 - t0);
+    const int j = c / (kHeadDim / 8);
+    const int d0 = (c % (kHeadDim / 8)) * 8;
+    float4* dst = reinterpret_cast<float4*>(reps + (static_cast<int64_t>(j) * nb + b) * kHeadDim + d0);
+    dst[0] = make_float4(acc[0] / cnt, acc[1] / cnt, acc[2] / cnt, acc[3] / cnt);
+    dst[1] = make_float4(acc[4] / cnt, acc[5] / cnt, acc[6] / cnt, acc[7] / cnt);
+}
+
+// Partial sums of the multi-head queries of sub-chunk i over token split s
+// (split_len tokens). Grid (M, splits).
+__global__ void __launch_bounds__(512) k_fp_partial(const uint4* __restrict__ q, int64_t N, int D8,
+                                                     int L, int split_len, int splits,
+                                                     float* __restrict__ partial)
+{
+    const int64_t i = blockIdx.x;
+    const int s = blockIdx.y;
+    const int64_t sc0 = i * L;
+    const int64_t sc1 = (sc0 + L < N) ? sc0 + L : N;
+    const int64_t t0 = sc0 + static_cast<int64_t>(s) * split_len;
+    const int64_t t1 = (t0 + split_len < sc1) ? t0 + split_len : sc1;
+    float* dst_row = partial + (i * splits + s) * static_cast<int64_t>(D8) * 8;
+    for (int c = threadIdx.x; c < D8; c += blockDim.x) {
+        float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+        const uint4* src = q + c;
+        int64_t t = t0;
+        for (; t + 8 <= t1; t += 8) {
+            uint4 x[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) x[u] = ld_stream(src + (t + u) * D8);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) add_bf16x8(acc, x[u]);
+        }
+        for (; t < t1; ++t) add_bf16x8(acc, ld_stream(src + t * D8));
+        float4* dst = reinterpret_cast<float4*>(dst_row + c * 8);
+        dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+        dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    }
+}
+
+// Deterministic block-wide sum (fixed shuffle tree, fixed warp order).
+__device__ float block_sum(float v, float* red)
+{
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) red[w] = v;
+    __syncthreads();
+    float t = 0.f;
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < (blockDim.x + 31) / 32; ++i) t += red[i];
+        red[0] = t;
+    }
+    __syncthreads();
+    t = red[0];
+    __syncthreads();
+    return t;
+}
+
+// v_i = (sum of the partials in split order) / |X_i|, and ||v_i||_2.
+__global__ void __launch_bounds__(512) k_fp_finalize(const float* __restrict__ partial, int D,
+                                                      int splits, int L, int64_t N,
+                                                      float* __restrict__ fp,
+                                                      float* __restrict__ norms)
+{
+    __shared__ float red[32];
+    const int64_t i = blockIdx.x;
+    const int64_t cnt = ((i + 1) * L < N ? (i + 1) * L : N) - i * L;
+    const float inv_cnt = 1.0f / static_cast<float>(cnt);
+    float ss = 0.f;
+    for (int c = threadIdx.x; c < D; c += blockDim.x) {
+        float v = 0.f;
+        for (int s = 0; s < splits; ++s) v += partial[(i * splits + s) * D + c];
+        v = v * inv_cnt;
+        fp[i * D + c] = v;
+        ss += v * v;
+    }
+    ss = block_sum(ss, red);
+    if (threadIdx.x == 0) norms[i] = sqrtf(ss);
+}
+
+// gram[i][d] = cos(v_i, v_{i+d}) = v~_i . v~_{i+d} for 1 <= d < S_max and i+d
+// in the same outer chunk; 0 when either norm is 0. One warp per (i, d).
+__global__ void k_gram(const float* __restrict__ fp, const float* __restrict__ norms, int D, int M,
+                       int S_max, int per_outer, float* __restrict__ gram)
+{
+    const int i = blockIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nw = blockDim.x >> 5;
+    const int chunk_end = min(M, (i / per_outer + 1) * per_outer);
+    for (int d = warp + 1; d < S_max; d += nw) {
+        const int j = i + d;
+        if (j >= chunk_end) continue;
+        const float* a = fp + static_cast<int64_t>(i) * D;
+        const float* b = fp + static_cast<int64_t>(j) * D;
+        float s = 0.f;
+        for (int c = lane; c < D; c += 32) s = fmaf(a[c], b[c], s);
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+        if (lane == 0) {
+            const float na = norms[i], nb = norms[j];
+            gram[static_cast<int64_t>(i) * S_max + d] = (na > 0.f && nb > 0.f) ? s / (na * nb) : 0.f;
+        }
+    }
+}
+
+// Exclusive block scan of 0/1 flags; returns this thread's exclusive prefix,
+// *total receives the block total.
+__device__ int block_exclusive_scan(int f, int* sh, int* total)
+{
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+    int x = f;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) sh[w] = x;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int run = 0;
+        for (int i = 0; i < nw; ++i) {
+            const int t = sh[i];
+            sh[i] = run;
+            run += t;
+        }
+        sh[nw] = run;
+    }
+    __syncthreads();
+    const int excl = sh[w] + x - f;
+    *total = sh[nw];
+    __syncthreads();
+    return excl;
+}
+
+// Algorithm 1 in each outer chunk (one thread per chunk walks its sub-chunks:
+// the anchor a admits j while cos(v_a, v_j) >= theta and |C_a| < S_max), then
+// one block compacts the anchor flags into unit_start and n_units.
+__global__ void __launch_bounds__(1024) k_cluster(const float* __restrict__ gram, int M, int S_max,
+                                                  int per_outer, float theta,
+                                                  int32_t* __restrict__ flag,
+                                                  int32_t* __restrict__ unit_start,
+                                                  int32_t* __restrict__ n_units)
+{
+    __shared__ int sh[40];
+    const bool always = theta <= -1.0f;
+    const int n_chunks = (M + per_outer - 1) / per_outer;
+    for (int c = threadIdx.x; c < n_chunks; c += blockDim.x) {
+        const int c0 = c * per_outer;
+        const int c1 = min(M, c0 + per_outer);
+        int a = c0;
+        while (a < c1) {
+            flag[a] = 1;
+            int size = 1, j = a + 1;
+            while (j < c1 && size < S_max) {
+                const bool admit = always || gram[static_cast<int64_t>(a) * S_max + (j - a)] >= theta;
+                if (!admit) break;
+                flag[j] = 0;
+                ++size;
+                ++j;
+            }
+            a = j;
+        }
+    }
+    __syncthreads();
+    int offset = 0;
+    for (int base = 0; base < M; base += blockDim.x) {
+        const int i = base + threadIdx.x;
+        const int f = (i < M) ? flag[i] : 0;
+        int total;
+        const int excl = block_exclusive_scan(f, sh, &total);
+        if (f) unit_start[offset + excl] = i;
+        offset += total;
+    }
+    for (int i = offset + threadIdx.x; i <= M; i += blockDim.x) unit_start[i] = M;
+    if (threadIdx.x == 0) *n_units = offset;
+}
+
+}  // namespace
+
+cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, float* reps,
+                              float* fingerprints, int32_t* unit_start, int32_t* n_units,
+                              uint8_t* ws, cudaStream_t st)
+{
+    const WsLayout lay = ws_layout(d);
+    float* partial = reinterpret_cast<float*>(ws + lay.fp_partial);
+    float* norms = reinterpret_cast<float*>(ws + lay.norms);
+    float* gram = reinterpret_cast<float*>(ws + lay.gram);
+    int32_t* flag = reinterpret_cast<int32_t*>(ws + lay.anchor);
+
+    const int row_chunks = d.Hkv * (kHeadDim / 8);
+    k_block_reps<<<static_cast<unsigned>(d.nb), row_chunks, 0, st>>>(
+        static_cast<const uint4*>(k), d.N, row_chunks, d.B, d.nb, reps);
+
+    const int D8 = d.D / 8;
+    const int split_len = (d.L + d.fp_splits - 1) / d.fp_splits;
+    k_fp_partial<<<dim3(static_cast<unsigned>(d.M), d.fp_splits), D8 < 512 ? D8 : 512, 0, st>>>(
+        static_cast<const uint4*>(q), d.N, D8, d.L, split_len, d.fp_splits, partial);
+    k_fp_finalize<<<static_cast<unsigned>(d.M), 512, 0, st>>>(partial, d.D, d.fp_splits, d.L, d.N,
+                                                               fingerprints, norms);
+    if (d.S_max > 1) {
+        const int warps = d.S_max - 1 < 16 ? d.S_max - 1 : 16;
+        k_gram<<<static_cast<unsigned>(d.M), 32 * warps, 0, st>>>(fingerprints, norms, d.D,
+                                                                  static_cast<int>(d.M), d.S_max,
+                                                                  d.per_outer, gram);
+    }
+    k_cluster<<<1, 1024, 0, st>>>(gram, static_cast<int>(d.M), d.S_max, d.per_outer, d.theta, flag,
+                                  unit_start, n_units);
+    return cudaGetLastError();
+}
+
+}  // namespace scale

@@ -1,0 +1,127 @@
+// scale_internal.h -- definitions shared by the library's translation units:
+// derived sizes, workspace layout, launch helpers of the kernels and the
+// device-side unit table.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "../../include/scale.h"
+
+namespace scale {
+
+constexpr int kHeadDim = 128;
+constexpr int kSegRows = 64;         // rows of one K/V TMA box (a "segment")
+constexpr int kMaxSegments = 1024;   // distant segments per unit the attention kernel can hold
+constexpr int kStatusOffset = 0;     // device status word (int32) at the start of the workspace
+constexpr size_t kAlign = 256;
+
+// Device status word values: 0, SCALE_ERR_TIMEOUT, SCALE_ERR_DEVICE.
+
+struct Derived {
+    int64_t N;
+    int Hq, Hkv, g, dh;
+    int L;           // sub-chunk
+    int S_max;       // max sub-chunks per cluster
+    int per_outer;   // sub-chunks per outer chunk
+    int B;           // block size
+    int k;           // top-k
+    int n_sink, n_local;
+    int64_t M;       // sub-chunks
+    int64_t nb;      // blocks
+    int D;           // H_q * d_h
+    int fp_splits;   // token splits of the fingerprint reduction
+    float theta, sigma, attn_scale;
+};
+
+// Workspace regions (byte offsets from the workspace base).
+struct WsLayout {
+    size_t status;      // int32 status word (+ padding)
+    size_t fp_partial;  // fp32 [M][fp_splits][D]
+    size_t norms;       // fp32 [M]
+    size_t gram;        // fp32 [M][S_max]   cosine of sub-chunk i with i+d
+    size_t anchor;      // int32 [M]         1 if sub-chunk i opens a cluster
+    size_t logits;      // fp32 [M][H_q][nb]
+    size_t stats;       // fp32 [M][H_q][2]  (row max, 1 / row sum)
+    size_t scores;      // fp32 [M][nb]
+    size_t total;
+};
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+int derive(const scale_params_t* p, Derived* d);
+WsLayout ws_layout(const Derived& d);
+
+// Unit table as the kernels see it.
+struct Units {
+    const int32_t* unit_start;  // SCR only
+    const int32_t* n_units;     // SCR only (device)
+    int per_subchunk;
+    int64_t N;
+    int L;
+    int M;
+};
+
+// Units starting in [tok_begin, tok_end): [first, first + count) with count
+// bounded by max_units; both modes.
+__device__ __forceinline__ int units_total(const Units& t)
+{
+    return t.per_subchunk ? t.M : *t.n_units;
+}
+
+// First unit whose first sub-chunk index is >= sc (binary search in SCR mode).
+__device__ __forceinline__ int unit_lower_bound(const Units& t, int sc)
+{
+    if (t.per_subchunk) return sc < t.M ? sc : t.M;
+    int lo = 0, hi = *t.n_units;
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (t.unit_start[mid] < sc) lo = mid + 1;
+        else hi = mid;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ void unit_range(const Units& t, int u, int* anchor, int64_t* s,
+                                           int64_t* e)
+{
+    int a, b;
+    if (t.per_subchunk) {
+        a = u;
+        b = u + 1;
+    } else {
+        a = t.unit_start[u];
+        b = t.unit_start[u + 1];
+    }
+    *anchor = a;
+    *s = static_cast<int64_t>(a) * t.L;
+    const int64_t ee = static_cast<int64_t>(b) * t.L;
+    *e = ee < t.N ? ee : t.N;
+}
+
+__device__ __forceinline__ void record_status(int32_t* status, int32_t code)
+{
+    atomicCAS(status, 0, code);
+}
+
+// ---- launchers (defined in the .cu files) ----
+cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, float* reps,
+                              float* fingerprints, int32_t* unit_start, int32_t* n_units,
+                              uint8_t* ws, cudaStream_t st);
+cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
+                          const float* reps, const float* fingerprints, const int32_t* unit_start,
+                          const int32_t* n_units, int32_t* sel_blocks, int32_t* sel_count,
+                          float* sel_scores, uint8_t* ws, cudaStream_t st);
+cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
+                                  const void* q, const void* k, const void* v,
+                                  const int32_t* unit_start, const int32_t* n_units,
+                                  const int32_t* sel_blocks, const int32_t* sel_count, void* out,
+                                  uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
+cudaError_t launch_wait_selftest(uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
+
+// Distant segments per unit the attention kernel may meet for these parameters.
+int64_t max_distant_segments(const Derived& d);
+
+}  // namespace scale

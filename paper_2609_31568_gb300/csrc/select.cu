@@ -1,0 +1,323 @@
+// select.cu -- steps (b) and (c) of the SCR prefill path: cluster-level
+// retrieval with head soft-voting (Eq. 9, Sec. V-A3 "Selection function
+// instantiation") over block representative keys, then a deterministic top-k.
+//
+//   k_logits  z[u][h][b] = sigma * v_a(u)^(h) . r_b^(h/g)   (fp32 GEMM tile per KV head)
+//   k_stats   per (u, h): max_b z and 1 / sum_b exp(z - max) over the candidates
+//   k_vote    score[u][b] = sum_h exp(z[u][h][b] - max) / sum   (heads in order)
+//   k_topk    radix select of the k-th largest (score, -b) key, then an
+//             index-ordered compaction: output ascending, ties to the lower b.
+//
+// Candidates of unit u are the blocks with a token in [n_sink, W_u),
+// W_u = max(0, s_u - n_local): the contiguous range [b_lo, b_hi(u)).
+#include <cmath>
+
+#include "scale_internal.h"
+
+namespace scale {
+namespace {
+
+constexpr int kLogitUnitRows = 32;  // rows (unit, head) per logits tile
+constexpr int kLogitBlocks = 64;    // blocks per logits tile
+constexpr int kLogitThreads = 256;
+
+struct SelArgs {
+    Units ut;
+    int sc_begin, sc_end;  // sub-chunk range of units to process
+    int Hq, g;
+    int64_t nb;
+    int B, k, n_sink, n_local;
+    float sigma;
+};
+
+__device__ __forceinline__ void cand_range(const SelArgs& a, int64_t s, int64_t* lo, int64_t* hi)
+{
+    const int64_t W = s - a.n_local > 0 ? s - a.n_local : 0;
+    *lo = a.n_sink / a.B;                 // first block with (b+1)B > n_sink
+    *hi = (W + a.B - 1) / a.B;            // one past the last block with bB < W
+    if (*hi > a.nb) *hi = a.nb;
+    if (*hi < *lo) *hi = *lo;
+}
+
+// Grid: (unit tiles, block tiles, KV heads). Rows of the A tile are
+// (unit, query head of this KV head) pairs.
+__global__ void __launch_bounds__(kLogitThreads) k_logits(SelArgs a,
+                                                          const float* __restrict__ fp,
+                                                          const float* __restrict__ reps,
+                                                          float* __restrict__ logits)
+{
+    extern __shared__ float sm[];
+    float* As = sm;                                    // [rows][128]
+    float* Bs = sm + kLogitUnitRows * kHeadDim;        // [64][129]
+    const int units_per_tile = kLogitUnitRows / a.g;
+    const int rows = units_per_tile * a.g;
+    const int u_first = unit_lower_bound(a.ut, a.sc_begin);
+    const int u_end = unit_lower_bound(a.ut, a.sc_end);
+    const int u0 = u_first + blockIdx.x * units_per_tile;
+    if (u0 >= u_end) return;
+    const int j = blockIdx.z;
+    const int64_t b0 = static_cast<int64_t>(blockIdx.y) * kLogitBlocks;
+    const int D = a.Hq * kHeadDim;
+
+    // The tile is needed only if some unit's candidate range meets [b0, b0+64).
+    __shared__ int64_t s_lo[kLogitUnitRows], s_hi[kLogitUnitRows];
+    __shared__ int s_anchor[kLogitUnitRows];
+    __shared__ int any;
+    if (threadIdx.x == 0) any = 0;
+    __syncthreads();
+    if (threadIdx.x < units_per_tile) {
+        const int u = u0 + threadIdx.x;
+        int64_t lo = 0, hi = 0;
+        int anc = 0;
+        if (u < u_end) {
+            int64_t s, e;
+            unit_range(a.ut, u, &anc, &s, &e);
+            cand_range(a, s, &lo, &hi);
+        }
+        s_lo[threadIdx.x] = lo;
+        s_hi[threadIdx.x] = hi;
+        s_anchor[threadIdx.x] = anc;
+        if (lo < hi && lo < b0 + kLogitBlocks && hi > b0) atomicOr(&any, 1);
+    }
+    __syncthreads();
+    if (!any) return;
+
+    for (int i = threadIdx.x; i < rows * kHeadDim; i += blockDim.x) {
+        const int r = i / kHeadDim, d = i % kHeadDim;
+        const int ul = r / a.g;
+        const int h = j * a.g + r % a.g;
+        As[i] = (u0 + ul < u_end) ? fp[static_cast<int64_t>(s_anchor[ul]) * D + h * kHeadDim + d] : 0.f;
+    }
+    for (int i = threadIdx.x; i < kLogitBlocks * kHeadDim; i += blockDim.x) {
+        const int bb = i / kHeadDim, d = i % kHeadDim;
+        const int64_t b = b0 + bb;
+        Bs[bb * (kHeadDim + 1) + d] = (b < a.nb) ? reps[(static_cast<int64_t>(j) * a.nb + b) * kHeadDim + d] : 0.f;
+    }
+    __syncthreads();
+
+    const int tx = threadIdx.x % kLogitBlocks;
+    const int ty = threadIdx.x / kLogitBlocks;
+    const int64_t b = b0 + tx;
+    const float* bp = Bs + tx * (kHeadDim + 1);
+    for (int r = ty; r < rows; r += kLogitThreads / kLogitBlocks) {
+        const int ul = r / a.g;
+        if (u0 + ul >= u_end || b < s_lo[ul] || b >= s_hi[ul]) continue;
+        const float* ap = As + r * kHeadDim;
+        float acc = 0.f;
+#pragma unroll 8
+        for (int d = 0; d < kHeadDim; ++d) acc = fmaf(ap[d], bp[d], acc);
+        const int h = j * a.g + r % a.g;
+        logits[(static_cast<int64_t>(u0 + ul) * a.Hq + h) * a.nb + b] = a.sigma * acc;
+    }
+}
+
+// One warp per (unit, head): row max and 1 / sum of exp(z - max) over the candidates.
+__global__ void __launch_bounds__(256) k_stats(SelArgs a, const float* __restrict__ logits,
+                                               float* __restrict__ stats)
+{
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int u_first = unit_lower_bound(a.ut, a.sc_begin);
+    const int u_end = unit_lower_bound(a.ut, a.sc_end);
+    const int64_t uh = static_cast<int64_t>(blockIdx.x) * 8 + warp;
+    const int u = u_first + static_cast<int>(uh / a.Hq);
+    const int h = static_cast<int>(uh % a.Hq);
+    if (u >= u_end) return;
+    int anc;
+    int64_t s, e, lo, hi;
+    unit_range(a.ut, u, &anc, &s, &e);
+    cand_range(a, s, &lo, &hi);
+    if (lo >= hi) return;
+    const float* z = logits + (static_cast<int64_t>(u) * a.Hq + h) * a.nb;
+    float m = -INFINITY;
+    for (int64_t b = lo + lane; b < hi; b += 32) m = fmaxf(m, z[b]);
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+    float sum = 0.f;
+    for (int64_t b = lo + lane; b < hi; b += 32) sum += expf(z[b] - m);
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+    if (lane == 0) {
+        stats[(static_cast<int64_t>(u) * a.Hq + h) * 2] = m;
+        stats[(static_cast<int64_t>(u) * a.Hq + h) * 2 + 1] = 1.0f / sum;
+    }
+}
+
+// score[u][b] = sum over heads (in order) of exp(z - max) / sum; NaN off the candidates.
+__global__ void __launch_bounds__(256) k_vote(SelArgs a, const float* __restrict__ logits,
+                                              const float* __restrict__ stats,
+                                              float* __restrict__ scores)
+{
+    const int u_first = unit_lower_bound(a.ut, a.sc_begin);
+    const int u_end = unit_lower_bound(a.ut, a.sc_end);
+    const int u = u_first + blockIdx.y;
+    if (u >= u_end) return;
+    const int64_t b = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (b >= a.nb) return;
+    int anc;
+    int64_t s, e, lo, hi;
+    unit_range(a.ut, u, &anc, &s, &e);
+    cand_range(a, s, &lo, &hi);
+    float score = __int_as_float(0x7FC00000);
+    if (b >= lo && b < hi) {
+        score = 0.f;
+        for (int h = 0; h < a.Hq; ++h) {
+            const int64_t uh = static_cast<int64_t>(u) * a.Hq + h;
+            score += expf(logits[uh * a.nb + b] - stats[uh * 2]) * stats[uh * 2 + 1];
+        }
+    }
+    scores[static_cast<int64_t>(u) * a.nb + b] = score;
+}
+
+// Order-preserving map of a float onto uint32 (larger float -> larger key).
+__device__ __forceinline__ uint32_t float_key(float f)
+{
+    const uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ int scan_excl(int f, int* sh, int* total)
+{
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int x = f;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) sh[w] = x;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int run = 0;
+        for (int i = 0; i < nw; ++i) {
+            const int t = sh[i];
+            sh[i] = run;
+            run += t;
+        }
+        sh[nw] = run;
+    }
+    __syncthreads();
+    const int r = sh[w] + x - f;
+    *total = sh[nw];
+    __syncthreads();
+    return r;
+}
+
+constexpr int kTopkThreads = 512;
+
+// One CTA per unit. The k-th largest key T is found with four 8-bit radix
+// passes; the selected blocks are those with key > T plus the lowest-indexed
+// ones with key == T, emitted in ascending block order.
+__global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* __restrict__ scores,
+                                                       int32_t* __restrict__ sel,
+                                                       int32_t* __restrict__ sel_count)
+{
+    __shared__ int hist[256];
+    __shared__ int sh[40];
+    __shared__ uint32_t s_prefix;
+    __shared__ int s_need;
+    const int u_first = unit_lower_bound(a.ut, a.sc_begin);
+    const int u_end = unit_lower_bound(a.ut, a.sc_end);
+    const int u = u_first + blockIdx.x;
+    if (u >= u_end) return;
+    int anc;
+    int64_t s, e, lo, hi;
+    unit_range(a.ut, u, &anc, &s, &e);
+    cand_range(a, s, &lo, &hi);
+    const int64_t n = hi - lo;
+    int32_t* out = sel + static_cast<int64_t>(u) * a.k;
+    const float* sc = scores + static_cast<int64_t>(u) * a.nb;
+
+    if (n <= a.k) {
+        for (int i = threadIdx.x; i < a.k; i += blockDim.x) out[i] = (i < n) ? static_cast<int32_t>(lo + i) : -1;
+        if (threadIdx.x == 0) sel_count[u] = static_cast<int32_t>(n);
+        return;
+    }
+    if (threadIdx.x == 0) {
+        s_prefix = 0;
+        s_need = a.k;
+    }
+    uint32_t mask = 0;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+        __syncthreads();
+        const uint32_t prefix = s_prefix;
+        for (int64_t b = lo + threadIdx.x; b < hi; b += blockDim.x) {
+            const uint32_t key = float_key(sc[b]);
+            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int need = s_need, cum = 0, d = 255;
+            for (; d > 0; --d) {
+                if (cum + hist[d] >= need) break;
+                cum += hist[d];
+            }
+            s_need = need - cum;
+            s_prefix = prefix | (static_cast<uint32_t>(d) << shift);
+        }
+        mask |= 255u << shift;
+        __syncthreads();
+    }
+    const uint32_t T = s_prefix;
+    const int need_eq = s_need;  // how many keys equal to T to take, lowest b first
+    int taken = 0, eq_seen = 0;
+    for (int64_t base = lo; base < hi; base += blockDim.x) {
+        const int64_t b = base + threadIdx.x;
+        const uint32_t key = (b < hi) ? float_key(sc[b]) : 0u;
+        const int is_eq = (b < hi) && key == T;
+        int eq_total;
+        const int eq_rank = eq_seen + scan_excl(is_eq, sh, &eq_total);
+        const int pick = (b < hi) && (key > T || (is_eq && eq_rank < need_eq));
+        int pick_total;
+        const int pos = taken + scan_excl(pick, sh, &pick_total);
+        if (pick) out[pos] = static_cast<int32_t>(b);
+        taken += pick_total;
+        eq_seen += eq_total;
+    }
+    for (int i = taken + threadIdx.x; i < a.k; i += blockDim.x) out[i] = -1;
+    if (threadIdx.x == 0) sel_count[u] = taken;
+}
+
+}  // namespace
+
+cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
+                          const float* reps, const float* fingerprints, const int32_t* unit_start,
+                          const int32_t* n_units, int32_t* sel_blocks, int32_t* sel_count,
+                          float* sel_scores, uint8_t* ws, cudaStream_t st)
+{
+    const WsLayout lay = ws_layout(d);
+    float* logits = reinterpret_cast<float*>(ws + lay.logits);
+    float* stats = reinterpret_cast<float*>(ws + lay.stats);
+    float* scores = sel_scores ? sel_scores : reinterpret_cast<float*>(ws + lay.scores);
+
+    SelArgs a;
+    a.ut = Units{unit_start, n_units, mode == SCALE_MODE_PER_SUBCHUNK, d.N, d.L, static_cast<int>(d.M)};
+    a.sc_begin = static_cast<int>(tok_begin / d.L);
+    a.sc_end = static_cast<int>((tok_end + d.L - 1) / d.L);
+    a.Hq = d.Hq;
+    a.g = d.g;
+    a.nb = d.nb;
+    a.B = d.B;
+    a.k = d.k;
+    a.n_sink = d.n_sink;
+    a.n_local = d.n_local;
+    a.sigma = d.sigma;
+    const int max_units = a.sc_end - a.sc_begin;  // units in range <= sub-chunks in range
+    if (max_units <= 0) return cudaSuccess;
+
+    const int upt = kLogitUnitRows / d.g;
+    const size_t smem = (kLogitUnitRows * kHeadDim + kLogitBlocks * (kHeadDim + 1)) * sizeof(float);
+    static bool attr = false;
+    if (!attr) {
+        cudaError_t e = cudaFuncSetAttribute(k_logits, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        attr = true;
+    }
+    dim3 gl((max_units + upt - 1) / upt, static_cast<unsigned>((d.nb + kLogitBlocks - 1) / kLogitBlocks), d.Hkv);
+    k_logits<<<gl, kLogitThreads, smem, st>>>(a, fingerprints, reps, logits);
+    const int64_t rows = static_cast<int64_t>(max_units) * d.Hq;
+    k_stats<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a, logits, stats);
+    k_vote<<<dim3(static_cast<unsigned>((d.nb + 255) / 256), max_units), 256, 0, st>>>(a, logits, stats, scores);
+    k_topk<<<max_units, kTopkThreads, 0, st>>>(a, scores, sel_blocks, sel_count);
+    return cudaGetLastError();
+}
+
+}  // namespace scale

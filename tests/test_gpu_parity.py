@@ -1,0 +1,299 @@
+"""GPU parity of every step of the SCR path against the CPU fp64 oracle.
+
+All calls go through the C ABI (libscale.so via the ctypes binding). Inputs
+are the seeded synthetic tensors of ``synth``; expected values come from
+``oracle`` only.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_31568_gb300 as pkg
+from paper_2609_31568_gb300 import scale as S
+from _util import (ATTN_MAX_ABS, ATTN_MEAN_ABS, NEAR_TIE_GAP, attn_errors, compare_selection,
+                   inputs, sample_rows, to_f64_bf16)
+
+pytestmark = pytest.mark.gpu
+
+PER_CLUSTER, PER_SUB = S.SCALE_MODE_PER_CLUSTER, S.SCALE_MODE_PER_SUBCHUNK
+
+# Small cases that span several tiles and end in ragged pieces.
+RAGGED = dict(n_tokens=3000, block_size=48, n_sink=40, n_local=100, top_k=6)
+GQA_SMALL = dict(n_tokens=8192 + 333, sub_chunk=512, max_cluster_subchunks=4, outer_chunk=2048,
+                 top_k=8)
+
+
+@pytest.fixture(scope="session", autouse=True)
+def _built():
+    pkg.build()
+    S.load()
+
+
+def gpu_path(w, mode, dev, want_scores=True, **over):
+    p = S.params_for(w, **over)
+    buf = S.allocate(p, mode, want_scores=want_scores)
+    S.run_path(p, mode, *dev, buf)
+    torch.cuda.synchronize()
+    assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
+    return p, buf
+
+
+def oracle_path(w, q, k, v, mode, rows=None, **over):
+    ww = w.replace(**over) if over else w
+    return oracle.run_path(ww, q, k, v, per_subchunk=(mode == PER_SUB), rows=rows)
+
+
+def unit_count(buf, mode, w):
+    return w.n_subchunks if mode == PER_SUB else int(buf.n_units.item())
+
+
+# --------------------------------------------------------------------------- step (a)
+
+
+@pytest.mark.parametrize("name,over", [("gqa4-4k", {}), ("gqa4-4k", RAGGED),
+                                       ("llama8b-32k", GQA_SMALL), ("llama8b-32k", {})])
+def test_build_reps_parity(name, over):
+    w, q, k, v, dev = inputs(name, **over)
+    p, buf = gpu_path(w, PER_CLUSTER, dev)
+    ref = oracle_path(w, q, k, v, PER_CLUSTER)
+    reps = buf.reps.cpu().numpy().astype(np.float64)
+    np.testing.assert_allclose(reps, ref["reps"], rtol=0, atol=2e-5)
+    fp = buf.fingerprints.cpu().numpy().astype(np.float64)
+    np.testing.assert_allclose(fp, ref["fingerprints"], rtol=0, atol=2e-5)
+    n = int(buf.n_units.item())
+    assert buf.unit_start[: n + 1].cpu().numpy().tolist() == ref["unit_start"].tolist()
+    assert np.all(buf.unit_start[n + 1:].cpu().numpy() == w.n_subchunks)
+
+
+def _robust_theta(fp: np.ndarray, norms: np.ndarray, w) -> float:
+    """A threshold between observed anchor-candidate cosines, far (>1e-4) from all of them."""
+    vt = fp / norms[:, None]
+    per = w.outer_chunk // w.sub_chunk
+    cs = []
+    for i in range(len(vt)):
+        for d in range(1, w.max_cluster_subchunks):
+            j = i + d
+            if j < len(vt) and j // per == i // per:
+                cs.append(float(vt[i] @ vt[j]))
+    cs = np.sort(np.array(cs))
+    mid = len(cs) // 2
+    gaps = np.diff(cs)
+    window = range(max(0, mid - len(cs) // 4), min(len(gaps), mid + len(cs) // 4 + 1))
+    best = max(window, key=lambda i: gaps[i])
+    assert gaps[best] > 2e-4
+    return float(cs[best] + gaps[best] / 2)
+
+
+@pytest.mark.parametrize("name,over", [("gqa4-4k", dict(max_cluster_subchunks=4)),
+                                       ("llama8b-32k", GQA_SMALL)])
+def test_threshold_clustering_parity(name, over):
+    w, q, k, v, dev = inputs(name, **over)
+    fp, norms = oracle.fingerprints(q, w.sub_chunk)
+    theta = _robust_theta(fp, norms, w)
+    ref_us, margin = oracle.anchor_clustering(fp, norms, w.max_cluster_subchunks,
+                                              w.outer_chunk // w.sub_chunk, theta)
+    assert margin > 1e-4
+    p, buf = gpu_path(w, PER_CLUSTER, dev, theta=theta)
+    n = int(buf.n_units.item())
+    got = buf.unit_start[: n + 1].cpu().numpy()
+    assert got.tolist() == ref_us.tolist()
+    assert 1 < n < w.n_subchunks or len(ref_us) - 1 == n
+
+
+# --------------------------------------------------------------------------- steps (b), (c)
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+@pytest.mark.parametrize("name,over", [("gqa4-4k", {}), ("gqa4-4k", RAGGED),
+                                       ("llama8b-32k", {}), ("llama8b-128k", {})])
+def test_select_parity(name, over, mode):
+    w, q, k, v, dev = inputs(name, **over)
+    p, buf = gpu_path(w, mode, dev)
+    ref = oracle.run_path(w, q, k, v, per_subchunk=(mode == PER_SUB))
+    n = unit_count(buf, mode, w)
+    assert n == len(ref["sel_count"])
+    sel = buf.sel_blocks.cpu().numpy()[:n, : w.top_k]
+    cnt = buf.sel_count.cpu().numpy()[:n]
+    same, near = compare_selection(sel, cnt, ref)
+    # the soft-vote scores themselves, on the candidates
+    ref_sc = oracle.select(num_q_heads=w.num_q_heads, n_tokens=w.n_tokens, sub_chunk=w.sub_chunk,
+                           block_size=w.block_size, top_k=w.top_k, n_sink=w.n_sink,
+                           n_local=w.n_local, select_scale=1.0, per_subchunk=(mode == PER_SUB),
+                           reps=ref["reps"], v=ref["fingerprints"], unit_start=ref["unit_start"],
+                           want_scores=True)["scores"]
+    got_sc = buf.sel_scores.cpu().numpy()[:n].astype(np.float64)
+    cand = ~np.isnan(ref_sc)
+    assert np.array_equal(cand, ~np.isnan(got_sc))
+    np.testing.assert_allclose(got_sc[cand], ref_sc[cand], rtol=2e-5, atol=1e-6)
+    print(f"{name} mode={mode}: {n} units, {int((cnt > 0).sum())} retrievals, "
+          f"{near} near-tie units differ (gap < {NEAR_TIE_GAP})")
+
+
+# --------------------------------------------------------------------------- step (d)
+
+
+def _prefill_on(w, mode, dev, unit_start, n_units, sel, cnt, **over):
+    p = S.params_for(w, **over)
+    ws = torch.empty(S.scale_workspace_size(p, mode), dtype=torch.uint8, device="cuda")
+    S.scale_workspace_init(ws)
+    out = torch.zeros((w.n_tokens, w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    k = max(w.top_k, 1)
+    M = w.n_subchunks
+    sel_full = np.full((M, k), -1, np.int32)
+    cnt_full = np.zeros(M, np.int32)
+    sel_full[: sel.shape[0], : sel.shape[1]] = sel
+    cnt_full[: len(cnt)] = cnt
+    us = torch.from_numpy(np.ascontiguousarray(unit_start, np.int32)).cuda()
+    nu = torch.tensor([n_units], dtype=torch.int32, device="cuda")
+    S.scale_sparse_prefill(p, mode, 0, w.n_tokens, *dev, us, nu,
+                           torch.from_numpy(sel_full).cuda(), torch.from_numpy(cnt_full).cuda(), out, ws)
+    torch.cuda.synchronize()
+    assert S.scale_get_device_status(ws) == S.SCALE_OK
+    return out
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+@pytest.mark.parametrize("name,over,stride", [
+    ("gqa4-4k", {}, 1),
+    ("gqa4-4k", RAGGED, 1),
+    ("gqa4-4k", dict(top_k=0, n_sink=0), 1),
+    ("gqa4-4k", dict(block_size=256, top_k=2, n_sink=128, n_local=0), 1),
+    ("llama8b-32k", GQA_SMALL, 5),
+])
+def test_attention_parity_on_oracle_selection(name, over, stride, mode):
+    """scale_sparse_prefill on the oracle's selection vs the oracle's Eq. 10."""
+    w, q, k, v, dev = inputs(name, **over)
+    rows = np.arange(0, w.n_tokens, stride)
+    ref = oracle_path(w, q, k, v, mode, rows=rows)
+    us = ref["unit_start"] if mode == PER_CLUSTER else np.arange(w.n_subchunks + 1, dtype=np.int32)
+    out = _prefill_on(w, mode, dev, us, len(us) - 1, ref["sel"], ref["sel_count"])
+    got = to_f64_bf16(out[torch.from_numpy(rows).cuda()])
+    mx, mean = attn_errors(got, ref["attn"])
+    print(f"{name} {over} mode={mode}: max {mx:.3e} mean {mean:.3e}")
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+@pytest.mark.parametrize("name,n_random", [("llama8b-32k", 16), ("llama8b-128k", 8)])
+def test_end_to_end_parity_sampled(name, n_random, mode):
+    """All four steps on the GPU at the workload's full size; selection compared
+    unit by unit, attention on sampled rows of units whose selection matches."""
+    w, q, k, v, dev = inputs(name)
+    p, buf = gpu_path(w, mode, dev)
+    ref = oracle_path(w, q, k, v, mode)
+    n = unit_count(buf, mode, w)
+    sel = buf.sel_blocks.cpu().numpy()[:n, : w.top_k]
+    cnt = buf.sel_count.cpu().numpy()[:n]
+    same, near = compare_selection(sel, cnt, ref)
+    us = ref["unit_start"] if mode == PER_CLUSTER else np.arange(w.n_subchunks + 1, dtype=np.int32)
+    rows = sample_rows(w, us, n_random)
+    tok_us = np.minimum(us.astype(np.int64) * w.sub_chunk, w.n_tokens)
+    unit_of = np.searchsorted(tok_us, rows, side="right") - 1
+    rows = rows[same[unit_of]]
+    ref_attn = oracle.attention_rows(q=q, k=k, v=v, sub_chunk=w.sub_chunk, block_size=w.block_size,
+                                     top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                                     attn_scale=1.0 / np.sqrt(w.head_dim),
+                                     per_subchunk=(mode == PER_SUB), unit_start=ref["unit_start"],
+                                     sel=ref["sel"], sel_count=ref["sel_count"], rows=rows)
+    got = to_f64_bf16(buf.out[torch.from_numpy(rows).cuda()])
+    mx, mean = attn_errors(got, ref_attn)
+    print(f"{name} mode={mode}: {len(rows)} rows, max {mx:.3e} mean {mean:.3e}, {near} near-tie units")
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+# --------------------------------------------------------------------------- invariants
+
+
+def test_size_one_clusters_equal_per_subchunk_mode():
+    w, q, k, v, dev = inputs("gqa4-4k", max_cluster_subchunks=1)
+    _, a = gpu_path(w, PER_CLUSTER, dev)
+    _, b = gpu_path(w, PER_SUB, dev)
+    assert int(a.n_units.item()) == w.n_subchunks
+    assert torch.equal(a.sel_blocks, b.sel_blocks) and torch.equal(a.sel_count, b.sel_count)
+    assert torch.equal(a.out, b.out)
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+def test_outer_chunk_loop_equals_one_call(mode):
+    """Algorithm 2 runs per outer chunk; calling select + attention chunk by chunk
+    gives the same bits as one call over all tokens."""
+    w, q, k, v, dev = inputs("llama8b-32k", **GQA_SMALL)
+    p, whole = gpu_path(w, mode, dev)
+    buf = S.allocate(p, mode, want_scores=True)
+    S.scale_build_reps(p, dev[0], dev[1], buf.reps, buf.fingerprints, buf.unit_start, buf.n_units, buf.ws)
+    buf.out.zero_()
+    step = w.outer_chunk
+    for t0 in range(0, w.n_tokens, step):
+        t1 = min(w.n_tokens, t0 + step)
+        S.scale_select(p, mode, t0, t1, buf.reps, buf.fingerprints, buf.unit_start, buf.n_units,
+                       buf.sel_blocks, buf.sel_count, buf.sel_scores, buf.ws)
+        S.scale_sparse_prefill(p, mode, t0, t1, *dev, buf.unit_start, buf.n_units, buf.sel_blocks,
+                               buf.sel_count, buf.out, buf.ws)
+    torch.cuda.synchronize()
+    n = unit_count(whole, mode, w)
+    assert torch.equal(whole.sel_blocks[:n], buf.sel_blocks[:n])
+    assert torch.equal(whole.out, buf.out)
+
+
+def test_deterministic_bits():
+    w, q, k, v, dev = inputs("llama8b-32k", **GQA_SMALL)
+    _, a = gpu_path(w, PER_CLUSTER, dev)
+    _, b = gpu_path(w, PER_CLUSTER, dev)
+    n = int(a.n_units.item())
+    assert n == int(b.n_units.item())
+    # bit patterns (scores hold NaN off the candidates; rows past n_units are unused)
+    for x, y in ((a.reps, b.reps), (a.fingerprints, b.fingerprints), (a.unit_start, b.unit_start),
+                 (a.sel_blocks[:n], b.sel_blocks[:n]), (a.sel_count[:n], b.sel_count[:n]),
+                 (a.sel_scores[:n], b.sel_scores[:n]), (a.out, b.out)):
+        assert torch.equal(x.view(torch.int32) if x.dtype == torch.float32 else x,
+                           y.view(torch.int32) if y.dtype == torch.float32 else y)
+
+
+def test_prefill_host_matches_device_path():
+    w, q, k, v, dev = inputs("gqa4-4k", **RAGGED)
+    for mode in (PER_CLUSTER, PER_SUB):
+        p, buf = gpu_path(w, mode, dev, want_scores=False)
+        arena = torch.empty(S.scale_prefill_host_arena_size(p, mode), dtype=torch.uint8, device="cuda")
+        out = np.empty((w.n_tokens, w.num_q_heads, w.head_dim), np.uint16)
+        S.scale_prefill_host(p, mode, q, k, v, out, arena)
+        assert np.array_equal(out, buf.out.view(torch.int16).cpu().numpy().view(np.uint16))
+
+
+def test_wait_timeout_is_reported_and_context_survives():
+    w, q, k, v, dev = inputs("gqa4-4k")
+    p = S.params_for(w)
+    ws = torch.empty(S.scale_workspace_size(p, PER_CLUSTER), dtype=torch.uint8, device="cuda")
+    S.scale_workspace_init(ws)
+    S.scale_selftest_wait_timeout(ws, 1_000_000)  # 1 ms on a barrier nothing arrives at
+    assert S.scale_get_device_status(ws) == S.SCALE_ERR_TIMEOUT
+    S.scale_workspace_init(ws)
+    assert S.scale_get_device_status(ws) == S.SCALE_OK
+    _, buf = gpu_path(w, PER_CLUSTER, dev)  # the context is still usable
+    assert torch.isfinite(buf.out.float()).all()
+
+
+def test_invalid_arguments_are_rejected_before_launch():
+    w, q, k, v, dev = inputs("gqa4-4k")
+    p = S.params_for(w)
+    buf = S.allocate(p, PER_CLUSTER)
+    host_q = torch.from_numpy(q).view(torch.bfloat16)
+    with pytest.raises(S.ScaleError) as e:
+        S.scale_build_reps(p, host_q, dev[1], buf.reps, buf.fingerprints, buf.unit_start, buf.n_units, buf.ws)
+    assert e.value.rc == S.SCALE_ERR_INVALID_ARG
+    with pytest.raises(S.ScaleError) as e:
+        S.scale_select(p, PER_CLUSTER, 0, w.n_tokens, buf.reps, buf.fingerprints, buf.unit_start,
+                       buf.n_units, buf.sel_blocks, buf.sel_count, None, buf.ws[:1024])
+    assert e.value.rc == S.SCALE_ERR_WORKSPACE
+    with pytest.raises(S.ScaleError) as e:
+        S.scale_sparse_prefill(p, PER_CLUSTER, 100, w.n_tokens, *dev, buf.unit_start, buf.n_units,
+                               buf.sel_blocks, buf.sel_count, buf.out, buf.ws)
+    assert e.value.rc == S.SCALE_ERR_INVALID_ARG
+    odd = S.params_for(w, num_q_heads=3, num_kv_heads=1)
+    with pytest.raises(S.ScaleError) as e:
+        S.scale_sparse_prefill(odd, PER_SUB, 0, w.n_tokens, *dev, None, None, buf.sel_blocks,
+                               buf.sel_count, buf.out, buf.ws)
+    assert e.value.rc == S.SCALE_ERR_UNSUPPORTED
+    torch.cuda.synchronize()
+    assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
