@@ -121,6 +121,28 @@ int scale_build_reps(const scale_params_t *p, const void *q, const void *k, floa
                      float *fingerprints, int32_t *unit_start, int32_t *n_units, void *ws,
                      size_t ws_bytes, scale_stream_t stream);
 
+/* Step (a) without a workspace. The paper has no counterpart: this entry point
+ * exists for callers that cannot allocate device memory for the library, such
+ * as a host framework's plugin interface that hands over only input and output
+ * buffers, or a serving loop whose device memory pool is fully reserved and
+ * where a cudaMalloc (which may synchronise the device) is not allowed on the
+ * request path. It computes exactly what scale_build_reps computes, with the
+ * same arguments minus the workspace, and allocates nothing: its scratch is a
+ * fixed 16 MiB array inside the library, which every GPU that loads the
+ * library holds until the process exits.
+ *  - Limit: returns SCALE_ERR_WORKSPACE, without launching anything, when the
+ *    scratch step (a) needs for `p` exceeds 16 MiB (it grows with
+ *    M * ceil(L / 512) * H_q * 128 * 4 bytes; 4.2 MB for 128K tokens with
+ *    L = 2048, 32 MB for 1M tokens with L = 4096, which is rejected).
+ *  - Set-up: the first call on each device looks up the array's device address
+ *    with that device current; make that first call before any stream capture.
+ *  - Sharing: every call on a device uses the same array, which keeps the last
+ *    call's contents; calls whose work overlaps on the GPU (other streams, or
+ *    other host threads) race on it and must be serialised by the caller. */
+int scale_build_reps_noalloc(const scale_params_t *p, const void *q, const void *k, float *reps,
+                             float *fingerprints, int32_t *unit_start, int32_t *n_units,
+                             scale_stream_t stream);
+
 /* Steps (b) and (c). Eq. 9 with head soft-voting (Sec. V-A3): for every unit u
  * starting in [tok_begin, tok_end) (SCR: the clusters of unit_start; baseline:
  * the sub-chunks) with anchor sub-chunk a (its first), and every query head h:

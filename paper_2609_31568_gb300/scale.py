@@ -105,6 +105,7 @@ def load() -> ctypes.CDLL:
             "scale_workspace_size": [pp, i32, ctypes.POINTER(sz)],
             "scale_workspace_init": [P, sz, P],
             "scale_build_reps": [pp, P, P, P, P, P, P, P, sz, P],
+            "scale_build_reps_noalloc": [pp, P, P, P, P, P, P, P],
             "scale_select": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, sz, P],
             "scale_sparse_prefill": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, P, sz, P],
             "scale_get_device_status": [P, P, ctypes.POINTER(i32)],
@@ -187,6 +188,13 @@ def scale_build_reps(p, q, k, reps, fingerprints, unit_start, n_units, ws, strea
     _check("scale_build_reps", load().scale_build_reps(
         ctypes.byref(p), _ptr(q), _ptr(k), _ptr(reps), _ptr(fingerprints), _ptr(unit_start),
         _ptr(n_units), _ptr(ws), _nbytes(ws), _stream(stream)))
+
+
+def scale_build_reps_noalloc(p, q, k, reps, fingerprints, unit_start, n_units, stream=None) -> None:
+    """Step (a) with the library's fixed scratch array instead of a workspace."""
+    _check("scale_build_reps_noalloc", load().scale_build_reps_noalloc(
+        ctypes.byref(p), _ptr(q), _ptr(k), _ptr(reps), _ptr(fingerprints), _ptr(unit_start),
+        _ptr(n_units), _stream(stream)))
 
 
 def scale_select(p, mode, tok_begin, tok_end, reps, fingerprints, unit_start, n_units,

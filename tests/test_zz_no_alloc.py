@@ -1,0 +1,76 @@
+"""scale_build_reps_noalloc: step (a) for callers that cannot allocate.
+
+Such callers (a plugin interface that passes only input and output buffers, a
+serving loop whose device memory is fully reserved) cannot give the library a
+workspace; this entry point keeps its scratch in a fixed array inside the
+library instead. The test calls it through the C ABI twice in a row, on two
+different inputs (so the second call starts from the first call's leftover
+scratch), and checks each result against scale_build_reps, the entry point
+with a caller-provided workspace, within the tolerance of the other step (a)
+tests. It also checks that a problem needing more scratch than the fixed
+array is refused before anything is launched.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_31568_gb300 as pkg
+from paper_2609_31568_gb300 import scale as S
+from synth import generate_layer, workload
+
+pytestmark = pytest.mark.gpu
+
+REPS_FP_ATOL = 2e-5  # same bound as the step (a) parity tests
+
+
+def _outputs(p):
+    M = -(-p.n_tokens // p.sub_chunk)
+    nb = -(-p.n_tokens // p.block_size)
+    return (torch.empty((p.num_kv_heads, nb, 128), dtype=torch.float32, device="cuda"),
+            torch.empty((M, p.num_q_heads * 128), dtype=torch.float32, device="cuda"),
+            torch.empty(M + 1, dtype=torch.int32, device="cuda"),
+            torch.empty(1, dtype=torch.int32, device="cuda"))
+
+
+def _case(name, seed, **over):
+    w = workload(name, **over)
+    q, k, _ = generate_layer(w, seed=seed)
+    return w, torch.from_numpy(q).view(torch.bfloat16).cuda(), torch.from_numpy(k).view(torch.bfloat16).cuda()
+
+
+def test_noalloc_build_reps_matches_workspace_entry_point_twice():
+    pkg.build()
+    S.load()
+    cases = [_case("llama8b-32k", 3, n_tokens=16384 + 77, sub_chunk=1024, outer_chunk=4096,
+                   max_cluster_subchunks=4),
+             _case("gqa4-4k", 5, n_tokens=3000)]
+    for w, q, k in cases:
+        p = S.params_for(w)
+        ref = _outputs(p)
+        ws = torch.empty(S.scale_workspace_size(p, S.SCALE_MODE_PER_CLUSTER), dtype=torch.uint8, device="cuda")
+        S.scale_workspace_init(ws)
+        S.scale_build_reps(p, q, k, *ref, ws)
+        got = _outputs(p)
+        for x in got:
+            x.fill_(-7)  # any stale value must be overwritten
+        S.scale_build_reps_noalloc(p, q, k, *got)
+        torch.cuda.synchronize()
+        assert S.scale_get_device_status(ws) == S.SCALE_OK
+        np.testing.assert_allclose(got[0].cpu().numpy(), ref[0].cpu().numpy(), rtol=0, atol=REPS_FP_ATOL)
+        np.testing.assert_allclose(got[1].cpu().numpy(), ref[1].cpu().numpy(), rtol=0, atol=REPS_FP_ATOL)
+        assert torch.equal(got[3], ref[3])
+        n = int(ref[3].item())
+        assert torch.equal(got[2][: n + 1], ref[2][: n + 1])
+
+
+def test_noalloc_refuses_problems_beyond_its_scratch():
+    pkg.build()
+    S.load()
+    p = S.params_for(workload("llama8b-1m"))  # needs 32 MiB of step (a) scratch
+    small = torch.zeros(1024, dtype=torch.float32, device="cuda")
+    ints = torch.zeros(1024, dtype=torch.int32, device="cuda")
+    with pytest.raises(S.ScaleError) as e:
+        S.scale_build_reps_noalloc(p, small, small, small, small, ints, ints)
+    assert e.value.rc == S.SCALE_ERR_WORKSPACE
+    torch.cuda.synchronize()
