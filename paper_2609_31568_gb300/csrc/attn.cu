@@ -92,12 +92,13 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     __shared__ volatile int abort_flag;
     __shared__ int s_nseg;
 
-    // ---- work item: heaviest (last) query blocks first ----
+    // ---- work item: one cluster at a time (its distant K/V set stays in L2),
+    // heaviest (last) query blocks of the cluster first ----
     int lin = blockIdx.x;
     const int hp = lin % (a.Hkv * a.pairs);
     lin /= a.Hkv * a.pairs;
-    const int ul = lin % a.units_max;
-    const int qb = a.qb_max - 1 - lin / a.units_max;
+    const int qb = a.qb_max - 1 - lin % a.qb_max;
+    const int ul = lin / a.qb_max;
     const int kvh = hp / a.pairs;
     const int h0 = kvh * a.g + 2 * (hp % a.pairs);
 
