@@ -317,21 +317,19 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
         const uint32_t s_addr = lane_base + qt * 256;
         const uint32_t o_addr = s_addr + 128;
         float m_run = -INFINITY, l_run = 0.f;
-        float s[128];
         bool ok = true;
         for (int t = 0; t < T; ++t) {
             // tcgen05.ld/st are warp-collective: the outcome must be warp-uniform.
             const bool got = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.s_full[qt], t & 1, a.timeout_ns, &abort_flag));
             if (!got) { ok = false; break; }
             tc_fence_after();
+            // S row: four 32-column TMEM loads in flight, one wait.
+            uint32_t sr[128];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t v[32];
-                tmem_ld32(s_addr + c * 32, v);
-                tmem_ld_wait();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(v[i]);
-            }
+            for (int c = 0; c < 4; ++c)
+                tmem_ld32(s_addr + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
+            tmem_ld_wait();
+            float* s = reinterpret_cast<float*>(sr);
             if (t < n_dt) {
                 const int la = seg[2 * t].y, lb = seg[2 * t + 1].y;
                 if (la < 64 || lb < 64) {
@@ -348,9 +346,18 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                         if (c > lim) s[c] = -INFINITY;
                 }
             }
-            float mx = -INFINITY;
+            // Row max: eight independent three-input max chains.
+            float mx8[8];
 #pragma unroll
-            for (int c = 0; c < 128; ++c) mx = fmaxf(mx, s[c]);
+            for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+            for (int c = 8; c < 120; c += 16)
+#pragma unroll
+                for (int i = 0; i < 8; ++i) mx8[i] = fmax3(mx8[i], s[c + 2 * i], s[c + 2 * i + 1]);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[120 + i]);
+            const float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
+                                   fmaxf(mx8[6], mx8[7]));
             const float m_new = fmaxf(m_run, mx * a.scale_log2);
             if (m_new > m_run + kRescaleThreshold) {
                 const float alpha = ex2(m_run - m_new);
@@ -369,19 +376,25 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 m_run = m_new;
             }
             const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
-            float sum = 0.f;
+            // p = 2^(s * scale_log2 - m): packed FMA, then the exponential.
+            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
                 uint32_t pk[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
-                    const float p0 = ex2(fmaf(s[h * 64 + 2 * i], a.scale_log2, neg_m));
-                    const float p1 = ex2(fmaf(s[h * 64 + 2 * i + 1], a.scale_log2, neg_m));
-                    sum += p0 + p1;
-                    pk[i] = pack_bf16x2(p0, p1);
+                    float x0, x1;
+                    ffma2(x0, x1, s[h * 64 + 2 * i], s[h * 64 + 2 * i + 1], a.scale_log2, a.scale_log2,
+                          neg_m, neg_m);
+                    x0 = ex2(x0);
+                    x1 = ex2(x1);
+                    const int j = (i & 3) * 2;
+                    fadd2(acc[j], acc[j + 1], acc[j], acc[j + 1], x0, x1);
+                    pk[i] = pack_bf16x2(x0, x1);
                 }
                 tmem_st32(s_addr + h * 32, pk);
             }
+            const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
             l_run += sum;
             tmem_st_wait();
             tc_fence_before();
