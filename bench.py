@@ -401,10 +401,135 @@ def run_scale(args):
     return 0
 
 
+def run_stack(args):
+    """Multi-layer workload: attention-only TTFT of a chunked prefill over all layers.
+
+    Per step: scale_build_reps for every layer, then for each outer chunk (in
+    order) and each layer, scale_select and scale_sparse_prefill restricted to
+    that chunk's tokens -- the dependency order of a real chunked prefill."""
+    import torch
+
+    world, rank, local = dist_setup(args)
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    import paper_2609_31568_gb300 as pkg
+    from paper_2609_31568_gb300 import scale as S
+
+    pkg.build()
+    S.load()
+    w = workload(args.workload)
+    p = S.params_for(w)
+    stream = torch.cuda.current_stream()
+    layers = []
+    for l in range(w.layers):
+        q, k, v = generate_layer(w, layer=l, seed=w.seed + l + 1000 * rank)
+        layers.append([torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)])
+        del q, k, v
+    chunks = [(t0, min(w.n_tokens, t0 + w.outer_chunk)) for t0 in range(0, w.n_tokens, w.outer_chunk)]
+
+    def measure(mode, steps, warmup):
+        bufs = [pkg.allocate(p, mode) for _ in layers]
+        n_attn = len(chunks) * len(layers)
+
+        def step(ev=None):
+            for dev, b in zip(layers, bufs):
+                S.scale_build_reps(p, dev[0], dev[1], b.reps, b.fingerprints, b.unit_start, b.n_units, b.ws, stream)
+            i = 0
+            for t0, t1 in chunks:
+                for dev, b in zip(layers, bufs):
+                    S.scale_select(p, mode, t0, t1, b.reps, b.fingerprints, b.unit_start, b.n_units,
+                                   b.sel_blocks, b.sel_count, None, b.ws, stream)
+                    if ev is not None:
+                        ev[i][0].record(stream)
+                    S.scale_sparse_prefill(p, mode, t0, t1, *dev, b.unit_start, b.n_units, b.sel_blocks,
+                                           b.sel_count, b.out, b.ws, stream)
+                    if ev is not None:
+                        ev[i][1].record(stream)
+                    i += 1
+
+        for _ in range(warmup):
+            step()
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        clocks = ClockSampler(torch.cuda.current_device())
+        clocks.start()
+        evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(n_attn)] for _ in range(steps)]
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for i in range(steps):
+            step(evs[i])
+        end.record(stream)
+        torch.cuda.synchronize()
+        clk = clocks.stop()
+        if world > 1:
+            torch.distributed.barrier()
+        ms = start.elapsed_time(end) / steps
+        attn_ms = sum(e[0].elapsed_time(e[1]) for ev in evs for e in ev) / steps
+        for b in bufs:
+            st = S.scale_get_device_status(b.ws)
+            if st != S.SCALE_OK:
+                raise RuntimeError(f"device status {st}: {S.status_string(st)}")
+        per_sub = mode == S.SCALE_MODE_PER_SUBCHUNK
+        keys, calls, units = 0, 0, 0
+        for b in bufs:
+            n = w.n_subchunks if per_sub else int(b.n_units.item())
+            us = b.unit_start.cpu().numpy()
+            keys += key_counts(w, us, n, b.sel_blocks.cpu().numpy(), b.sel_count.cpu().numpy(), per_sub)
+            units += n
+            calls += S.scale_retrieval_calls(p, mode, None if per_sub else us[: n + 1], n)[1]
+        del bufs
+        return ms, attn_ms, clk, 4.0 * w.head_dim * w.num_q_heads * keys, calls, units
+
+    mode = S.SCALE_MODE_PER_SUBCHUNK if args.mode == "subchunk" else S.SCALE_MODE_PER_CLUSTER
+    ms, attn_ms, clk, flops, calls, units = measure(mode, args.steps, args.warmup)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    peaks = load_peaks()
+    achieved = flops / (attn_ms / 1e3) / 1e12
+    line = {
+        "metric": METRIC, "value": world * w.n_tokens / (ms / 1e3), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "ttft_ms": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": w.name, "n_tokens": w.n_tokens, "layers": w.layers, "mode": args.mode,
+                   "outer_chunk": w.outer_chunk, "loop": "chunk-major: every layer per outer chunk",
+                   "parallelism": f"independent stacks x{world}", "l2": "inputs larger than L2"},
+        "stages_ms": {"sparse_attention_total": attn_ms, "other": ms - attn_ms},
+        "retrieval_calls": calls, "units": units,
+        "roofline": {"bound": "tensor", "kernel": "k_sparse_attn", "achieved": achieved,
+                     "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
+                     "frac": achieved / peaks["bf16_sustained"], "frac_of_burst": achieved / peaks["bf16"],
+                     "peak_source": f"bf16 sustained, of {peaks['source']}",
+                     "algorithmic_flops_per_step": flops, "traffic": None},
+        "gpu_launches": args.steps * w.layers * (5 + len(chunks) * 5),
+        "clocks": clk,
+    }
+    if not args.no_baseline_mode and rank == 0:
+        other = S.SCALE_MODE_PER_SUBCHUNK if mode == S.SCALE_MODE_PER_CLUSTER else S.SCALE_MODE_PER_CLUSTER
+        ms2, attn2, _, flops2, calls2, units2 = measure(other, max(2, args.steps // 2), 1)
+        line["other_mode"] = {"mode": "subchunk" if other == S.SCALE_MODE_PER_SUBCHUNK else "cluster",
+                              "ms_per_step": ms2, "tokens_per_s": w.n_tokens / (ms2 / 1e3),
+                              "sparse_attention_ms": attn2, "retrieval_calls": calls2, "units": units2,
+                              "attn_tflops": flops2 / (attn2 / 1e3) / 1e12}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if workload(args.workload).layers > 1:
+        return run_stack(args)
     return run_scale(args)
 
 

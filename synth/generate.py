@@ -187,9 +187,21 @@ def generate_layer(w: Workload, layer: int = 0, seed: int | None = None,
     if workers is None:
         workers = min(len(jobs), os.cpu_count() or 1) if T * w.num_q_heads >= (1 << 20) else 1
     if workers > 1 and len(jobs) > 1:
+        import concurrent.futures as cf
         import multiprocessing as mp
-        with mp.get_context("spawn").Pool(workers) as pool:
-            parts = pool.map(_chunk_job, jobs, chunksize=1)
+
+        # A process pool that raises (BrokenProcessPool) if a worker dies,
+        # instead of waiting forever for its lost task.
+        with cf.ProcessPoolExecutor(max_workers=min(workers, 16),
+                                    mp_context=mp.get_context("spawn")) as ex:
+            for ch, (cq, ck, cv) in zip(range(c0, c1), ex.map(_chunk_job, jobs)):
+                a = max(t0, ch * CHUNK)
+                b = min(t1, ch * CHUNK + cq.shape[0])
+                s = a - ch * CHUNK
+                q[a - t0:b - t0] = cq[s:s + b - a]
+                k[a - t0:b - t0] = ck[s:s + b - a]
+                v[a - t0:b - t0] = cv[s:s + b - a]
+        return q, k, v
     else:
         cents = _centroids(w, layer, seed)
         parts = (_chunk(w, layer, seed, cents, ch) for ch in range(c0, c1))

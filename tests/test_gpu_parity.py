@@ -297,3 +297,55 @@ def test_invalid_arguments_are_rejected_before_launch():
     assert e.value.rc == S.SCALE_ERR_UNSUPPORTED
     torch.cuda.synchronize()
     assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
+
+
+# --------------------------------------------------------------------------- full-size stack and 1M
+
+
+def _full_size_check(w, q, k, v, mode, n_random, seed=7):
+    import time
+
+    t0 = time.time()
+    log = lambda *a: print(f"  [{time.time() - t0:6.1f}s]", *a, flush=True)  # noqa: E731
+    dev = [torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)]
+    p, buf = gpu_path(w, mode, dev, want_scores=False)
+    log("gpu path done")
+    ref = oracle_path(w, q, k, v, mode)
+    log("oracle selection done")
+    n = unit_count(buf, mode, w)
+    sel = buf.sel_blocks.cpu().numpy()[:n, : w.top_k]
+    cnt = buf.sel_count.cpu().numpy()[:n]
+    same, near = compare_selection(sel, cnt, ref)
+    us = ref["unit_start"] if mode == PER_CLUSTER else np.arange(w.n_subchunks + 1, dtype=np.int32)
+    rng = np.random.default_rng(seed)
+    tok_us = np.minimum(us.astype(np.int64) * w.sub_chunk, w.n_tokens)
+    rows = [int(tok_us[u]) for u in range(len(us) - 1)] + [int(tok_us[u + 1]) - 1 for u in range(len(us) - 1)]
+    rows += rng.integers(0, w.n_tokens, size=n_random).tolist()
+    rows = np.unique(np.array(rows, np.int64))
+    unit_of = np.searchsorted(tok_us, rows, side="right") - 1
+    rows = rows[same[unit_of]]
+    log(f"oracle attention on {len(rows)} rows")
+    ref_attn = oracle.attention_rows(q=q, k=k, v=v, sub_chunk=w.sub_chunk, block_size=w.block_size,
+                                     top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                                     attn_scale=1.0 / np.sqrt(w.head_dim),
+                                     per_subchunk=(mode == PER_SUB), unit_start=ref["unit_start"],
+                                     sel=ref["sel"], sel_count=ref["sel_count"], rows=rows)
+    log("oracle attention done")
+    got = to_f64_bf16(buf.out[torch.from_numpy(rows).cuda()])
+    mx, mean = attn_errors(got, ref_attn)
+    del buf, dev
+    torch.cuda.empty_cache()
+    return len(rows), mx, mean, near
+
+
+@pytest.mark.parametrize("layer", [0, 15, 31])
+def test_stack_64k_layers_full_size(layer):
+    """The 32-layer 64K stack: independent inputs per layer (seed = layer); layers 0, 15, 31."""
+    from synth import generate_layer, workload
+
+    w = workload("llama8b-64k-32l")
+    q, k, v = generate_layer(w, layer=layer)
+    for mode in (PER_CLUSTER, PER_SUB):
+        n, mx, mean, near = _full_size_check(w, q, k, v, mode, n_random=48, seed=layer)
+        print(f"layer {layer} mode={mode}: {n} rows, max {mx:.3e} mean {mean:.3e}, {near} near-tie units")
+        assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
