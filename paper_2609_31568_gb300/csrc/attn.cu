@@ -359,8 +359,12 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
             const float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
                                    fmaxf(mx8[6], mx8[7]));
             const float m_new = fmaxf(m_run, mx * a.scale_log2);
-            if (m_new > m_run + kRescaleThreshold) {
-                const float alpha = ex2(m_run - m_new);
+            const bool raise = m_new > m_run + kRescaleThreshold;
+            // The O rescale goes through warp-collective TMEM loads and stores,
+            // so the branch is taken by the whole warp when any row needs it;
+            // rows that do not keep their max and scale by 1.
+            if (__any_sync(0xFFFFFFFFu, raise)) {
+                const float alpha = raise ? ex2(m_run - m_new) : 1.0f;
                 l_run *= alpha;
                 if (t > 0) {
 #pragma unroll 1
@@ -373,7 +377,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                         tmem_st16(o_addr + c * 16, v);
                     }
                 }
-                m_run = m_new;
+                if (raise) m_run = m_new;
             }
             const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
             // p = 2^(s * scale_log2 - m): packed FMA, then the exponential.

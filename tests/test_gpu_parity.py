@@ -176,6 +176,32 @@ def test_attention_parity_on_oracle_selection(name, over, stride, mode):
 
 
 @pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+def test_attention_max_jump_in_alternate_rows(mode):
+    """Rows whose running max jumps in a later key tile next to rows whose max
+    does not: even rows get a large score against a few spike keys (the online
+    softmax of Sec. V-A3 must raise their max and rescale their partial sums),
+    odd rows score exactly 0 against them. Both kinds of row share each group
+    of 32 consecutive rows."""
+    w, q, k, v, _ = inputs("gqa4-4k")
+    q = q.copy()
+    k = k.copy()
+    spikes = np.arange(200, w.n_tokens, 512)
+    k[spikes] = 0
+    k[spikes, :, 0] = 0x4200  # bf16 32.0
+    q[0::2, :, 0] = 0x4100    # bf16 8.0: score 256 against a spike key
+    q[1::2, :, 0] = 0         # score 0 against a spike key
+    dev = [torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)]
+    rows = np.arange(w.n_tokens)
+    ref = oracle_path(w, q, k, v, mode, rows=rows)
+    us = ref["unit_start"] if mode == PER_CLUSTER else np.arange(w.n_subchunks + 1, dtype=np.int32)
+    out = _prefill_on(w, mode, dev, us, len(us) - 1, ref["sel"], ref["sel_count"])
+    got = to_f64_bf16(out)
+    mx, mean = attn_errors(got, ref["attn"])
+    print(f"mode={mode}: max {mx:.3e} mean {mean:.3e}")
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
 @pytest.mark.parametrize("name,n_random", [("llama8b-32k", 16), ("llama8b-128k", 8)])
 def test_end_to_end_parity_sampled(name, n_random, mode):
     """All four steps on the GPU at the workload's full size; selection compared
@@ -348,4 +374,17 @@ def test_stack_64k_layers_full_size(layer):
     for mode in (PER_CLUSTER, PER_SUB):
         n, mx, mean, near = _full_size_check(w, q, k, v, mode, n_random=48, seed=layer)
         print(f"layer {layer} mode={mode}: {n} rows, max {mx:.3e} mean {mean:.3e}, {near} near-tie units")
+        assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+def test_1m_context_full_size():
+    """The 1M-token layer, both modes: selection of every unit, attention on the
+    first and last row of every unit plus random rows."""
+    from synth import generate_layer, workload
+
+    w = workload("llama8b-1m")
+    q, k, v = generate_layer(w)
+    for mode in (PER_CLUSTER, PER_SUB):
+        n, mx, mean, near = _full_size_check(w, q, k, v, mode, n_random=40)
+        print(f"1M mode={mode}: {n} rows, max {mx:.3e} mean {mean:.3e}, {near} near-tie units")
         assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
