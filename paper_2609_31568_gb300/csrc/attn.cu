@@ -43,6 +43,13 @@ constexpr uint32_t kTileBytes = 128 * 128 * 2;  // one 128 x 128 bf16 tile
 constexpr uint32_t kHalf = kTileBytes / 2;    // one 64-column half (128 rows x 128 B)
 constexpr uint32_t kSegBytes = 64 * 128;      // one 64-row x 64-column box
 constexpr float kRescaleThreshold = 8.0f;     // log2 units
+// Softmax exponentials of column pair i go to the FMA pipe (exp2_poly2) when
+// bit (i % 8) is set, else to the special-function unit; the split balances
+// the two units, which otherwise bound the softmax.
+#ifndef SCALE_SOFT_EXP_MASK
+#define SCALE_SOFT_EXP_MASK 0x00
+#endif
+constexpr uint32_t kSoftExpMask = SCALE_SOFT_EXP_MASK;
 
 // Dynamic shared memory map (offsets from the 1024-aligned base).
 constexpr uint32_t kOffQ = 0;                          // 2 Q tiles
@@ -54,8 +61,9 @@ constexpr uint32_t kSmemBytes = kOffSeg + kMaxSegments * 8 + 1024;
 struct AttnArgs {
     Units ut;
     int sc_begin, sc_end;
-    int units_max;  // grid extent over units
-    int qb_max;     // grid extent over 128-row query blocks of one unit
+    int n_sc;       // sub-chunks in the token range
+    int qb_per_sc;     // 128-row query blocks per sub-chunk
+    int sc_per_chunk;  // sub-chunks per outer chunk
     int Hq, Hkv, g, pairs;
     int64_t N, nb;
     int B, k, n_sink, n_local;
@@ -92,24 +100,33 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     __shared__ volatile int abort_flag;
     __shared__ int s_nseg;
 
-    // ---- work item: one cluster at a time (its distant K/V set stays in L2),
-    // heaviest (last) query blocks of the cluster first ----
+    // ---- work item: a 128-row query block of one sub-chunk and a pair of
+    // query heads. The grid holds exactly the blocks of the sub-chunks in
+    // range (no idle CTAs whatever the clustering), outer chunk by outer
+    // chunk, so one cluster's distant K/V set is live in L2 at a time; within
+    // a chunk the last block comes first, which issues each cluster's
+    // heaviest rows (longest window) first. ----
     int lin = blockIdx.x;
     const int hp = lin % (a.Hkv * a.pairs);
     lin /= a.Hkv * a.pairs;
-    const int qb = a.qb_max - 1 - lin % a.qb_max;
-    const int ul = lin / a.qb_max;
     const int kvh = hp / a.pairs;
     const int h0 = kvh * a.g + 2 * (hp % a.pairs);
-
-    const int u = unit_lower_bound(a.ut, a.sc_begin) + ul;
-    if (u >= unit_lower_bound(a.ut, a.sc_end)) return;
+    const int per_chunk = a.sc_per_chunk * a.qb_per_sc;
+    const int c = lin / per_chunk;
+    const int sc0 = a.sc_begin + c * a.sc_per_chunk;
+    const int n_sc = (a.sc_end - sc0 < a.sc_per_chunk) ? a.sc_end - sc0 : a.sc_per_chunk;
+    const int idx = n_sc * a.qb_per_sc - 1 - (lin - c * per_chunk);
+    if (idx < 0) return;
+    const int sc = sc0 + idx / a.qb_per_sc;
+    const int u = unit_of_subchunk(a.ut, sc);
     int anchor;
     int64_t s_u, e_u;
     unit_range(a.ut, u, &anchor, &s_u, &e_u);
-    const int64_t q0 = s_u + static_cast<int64_t>(kRows) * qb;
-    if (q0 >= e_u) return;
-    const int64_t q_end = (q0 + kRows < e_u) ? q0 + kRows : e_u;
+    const int64_t sc_lo = static_cast<int64_t>(sc) * a.ut.L;
+    const int64_t sc_hi = (sc_lo + a.ut.L < e_u) ? sc_lo + a.ut.L : e_u;
+    const int64_t q0 = sc_lo + static_cast<int64_t>(kRows) * (idx % a.qb_per_sc);
+    if (q0 >= sc_hi) return;
+    const int64_t q_end = (q0 + kRows < sc_hi) ? q0 + kRows : sc_hi;
     const int64_t W = (s_u - a.n_local > 0) ? s_u - a.n_local : 0;
     const int n_lt = static_cast<int>((q_end - W + 127) / 128);
 
@@ -259,13 +276,14 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
             const uint32_t k_base = smem_addr(smem + kOffK);
             const uint32_t v_base = smem_addr(smem + kOffV);
             bool ok = mbar_wait_bounded(&bars.q_full, 0, a.timeout_ns, &abort_flag);
+            // Descriptors of the two stages differ by kTileBytes >> 4 in the address field.
+            constexpr uint64_t kStageStep = kTileBytes >> 4;
+            const uint64_t qdesc0 = sdesc_sw128(q_base, 16, 1024);
+            const uint64_t kdesc0 = sdesc_sw128(k_base, 16, 1024);
+            const uint64_t vdesc0 = sdesc_sw128(v_base, kHalf, 1024);
             auto issue_pv = [&](int t, int qt) {
-                const uint32_t vs = v_base + (t & 1) * kTileBytes;
-                const uint32_t d = tmem + qt * 256 + 128;
-                const uint32_t p = tmem + qt * 256;
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk)
-                    mma_ts(d, p + kk * 8, sdesc_sw128(vs + kk * 2048, kHalf, 1024), id_pv, (t > 0 || kk > 0) ? 1u : 0u);
+                mma_ts_k128<2048>(tmem + qt * 256 + 128, tmem + qt * 256, vdesc0 + (t & 1) * kStageStep, id_pv,
+                                  t > 0 ? 1u : 0u);
             };
             for (int t = 0; ok && t < T; ++t) {
                 const int st = t & 1;
@@ -279,12 +297,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                         tc_fence_after();
                         issue_pv(t - 1, qt);
                     }
-                    const uint32_t qs = q_base + qt * kTileBytes;
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
-                        mma_ss(tmem + qt * 256, sdesc_sw128(qs + off, 16, 1024), sdesc_sw128(ks + off, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
-                    }
+                    mma_ss_k128<kHalf>(tmem + qt * 256, qdesc0 + qt * kStageStep, kdesc0 + st * kStageStep, id_qk, 0u);
                     mma_commit(&bars.s_full[qt]);
                 }
                 if (!ok) break;
@@ -390,8 +403,12 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                     float x0, x1;
                     ffma2(x0, x1, s[h * 64 + 2 * i], s[h * 64 + 2 * i + 1], a.scale_log2, a.scale_log2,
                           neg_m, neg_m);
-                    x0 = ex2(x0);
-                    x1 = ex2(x1);
+                    if ((kSoftExpMask >> (i & 7)) & 1u) {
+                        exp2_poly2(x0, x1, x0, x1);
+                    } else {
+                        x0 = ex2(x0);
+                        x1 = ex2(x1);
+                    }
                     const int j = (i & 3) * 2;
                     fadd2(acc[j], acc[j + 1], acc[j], acc[j + 1], x0, x1);
                     pk[i] = pack_bf16x2(x0, x1);
@@ -479,10 +496,10 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
     a.ut = Units{unit_start, n_units, mode == SCALE_MODE_PER_SUBCHUNK, d.N, d.L, static_cast<int>(d.M)};
     a.sc_begin = static_cast<int>(tok_begin / d.L);
     a.sc_end = static_cast<int>((tok_end + d.L - 1) / d.L);
-    a.units_max = a.sc_end - a.sc_begin;
-    if (a.units_max <= 0) return cudaSuccess;
-    const int64_t unit_tokens = static_cast<int64_t>(mode == SCALE_MODE_PER_SUBCHUNK ? 1 : d.S_max) * d.L;
-    a.qb_max = static_cast<int>((unit_tokens + kRows - 1) / kRows);
+    a.n_sc = a.sc_end - a.sc_begin;
+    if (a.n_sc <= 0) return cudaSuccess;
+    a.qb_per_sc = static_cast<int>((d.L + kRows - 1) / kRows);
+    a.sc_per_chunk = d.per_outer;
     a.Hq = d.Hq;
     a.Hkv = d.Hkv;
     a.g = d.g;
@@ -503,7 +520,7 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
     cudaError_t e = cudaFuncSetAttribute(k_sparse_attn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(kSmemBytes));
     if (e != cudaSuccess) return e;
-    const int64_t grid = static_cast<int64_t>(a.units_max) * a.qb_max * d.Hkv * a.pairs;
+    const int64_t grid = static_cast<int64_t>(a.n_sc) * a.qb_per_sc * d.Hkv * a.pairs;
     if (grid <= 0 || grid > 0x7FFFFFFFll) return cudaErrorInvalidConfiguration;
     k_sparse_attn<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tq, tk, tv, a);
     return cudaGetLastError();

@@ -141,27 +141,69 @@ __device__ __forceinline__ void tc_fence_after()
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// D[tmem] (+)= A[smem desc] * B[smem desc]
-__device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                       uint32_t idesc, uint32_t accumulate)
+// Eight MMAs D (+)= A_j * B_j, j = 0..7, over one 128-deep K range held as two
+// 64-column halves of 128-byte-swizzled K-major tiles (A and B alike): the
+// descriptors of step j advance by 32 bytes per 16-element K step inside a
+// half and by `half_bytes` from the first half to the second. The first MMA
+// accumulates into D when `accumulate` != 0, the others always do.
+template <uint32_t half_bytes>
+__device__ __forceinline__ void mma_ss_k128(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate)
 {
+    constexpr uint64_t h = half_bytes >> 4;
     asm volatile(
-        "{\n\t.reg .pred p;\n\t"
+        "{\n\t.reg .pred p, q;\n\t.reg .b64 a, b;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        "setp.ne.b32 q, %5, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t"
+        "add.s64 a, %1, 2;\n\tadd.s64 b, %2, 2;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, 4;\n\tadd.s64 b, %2, 4;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, 6;\n\tadd.s64 b, %2, 6;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %6;\n\tadd.s64 b, %2, %6;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %7;\n\tadd.s64 b, %2, %7;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %8;\n\tadd.s64 b, %2, %8;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %9;\n\tadd.s64 b, %2, %9;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(1u), "n"(h), "n"(h + 2),
+        "n"(h + 4), "n"(h + 6)
         : "memory");
 }
 
-// D[tmem] (+)= A[tmem] * B[smem desc]
-__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                       uint32_t idesc, uint32_t accumulate)
+// Eight MMAs D (+)= A_j * B_j, j = 0..7, with A in TMEM (8 columns of packed
+// bf16 pairs = 16 K elements per step) and B an MN-major smem operand whose
+// descriptor advances by `step_bytes` per 16-element K step.
+template <uint32_t step_bytes>
+__device__ __forceinline__ void mma_ts_k128(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate)
 {
+    constexpr uint64_t st = step_bytes >> 4;
     asm volatile(
-        "{\n\t.reg .pred p;\n\t"
+        "{\n\t.reg .pred p, q;\n\t.reg .b64 b;\n\t.reg .b32 a;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        "setp.ne.b32 q, %5, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t"
+        "add.u32 a, %1, 8;\n\tadd.s64 b, %2, %6;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %3, q;\n\t"
+        "add.u32 a, %1, 16;\n\tadd.s64 b, %2, %7;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %3, q;\n\t"
+        "add.u32 a, %1, 24;\n\tadd.s64 b, %2, %8;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %3, q;\n\t"
+        "add.u32 a, %1, 32;\n\tadd.s64 b, %2, %9;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %3, q;\n\t"
+        "add.u32 a, %1, 40;\n\tadd.s64 b, %2, %10;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %3, q;\n\t"
+        "add.u32 a, %1, 48;\n\tadd.s64 b, %2, %11;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %3, q;\n\t"
+        "add.u32 a, %1, 56;\n\tadd.s64 b, %2, %12;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %3, q;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(1u), "n"(st), "n"(2 * st),
+        "n"(3 * st), "n"(4 * st), "n"(5 * st), "n"(6 * st), "n"(7 * st)
         : "memory");
 }
 
@@ -299,6 +341,32 @@ __device__ __forceinline__ void fadd2(float& d0, float& d1, float a0, float a1, 
         "add.rn.ftz.f32x2 x, x, y;\n\tmov.b64 {%0, %1}, x;\n\t}"
         : "=f"(d0), "=f"(d1)
         : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
+// (2^x0, 2^x1) on the FMA pipe, for softmax weights that are rounded to bf16
+// afterwards. Cody-Waite style split x = j + f with j = round(x) (adding
+// 1.5 * 2^23 rounds to an integer held in the low mantissa bits) and
+// |f| <= 1/2; 2^f from a degree-3 polynomial, the minimax fit of relative
+// error on [-1/2, 1/2] by the Remez exchange (fit_exp2.py beside these
+// sources; max relative error 7.5e-5 in fp32, against 2^-9 for the bf16
+// rounding that follows); 2^j is added into the exponent bits. Inputs below
+// -125 are raised to -125, so -inf gives 2^-125 instead of 0.
+__device__ __forceinline__ void exp2_poly2(float& r0, float& r1, float x0, float x1)
+{
+    constexpr float kRound = 12582912.0f;  // 1.5 * 2^23
+    constexpr float c0 = 0.9999280571937561f, c1 = 0.6932609677314758f;
+    constexpr float c2 = 0.2426111251115799f, c3 = 0.0551716685295105f;
+    x0 = fmaxf(x0, -125.0f);
+    x1 = fmaxf(x1, -125.0f);
+    float y0, y1, j0, j1, f0, f1, p0, p1;
+    fadd2(y0, y1, x0, x1, kRound, kRound);
+    fadd2(j0, j1, y0, y1, -kRound, -kRound);  // round(x), exact
+    ffma2(f0, f1, j0, j1, -1.0f, -1.0f, x0, x1);  // x - round(x), exact
+    ffma2(p0, p1, c3, c3, f0, f1, c2, c2);
+    ffma2(p0, p1, p0, p1, f0, f1, c1, c1);
+    ffma2(p0, p1, p0, p1, f0, f1, c0, c0);
+    r0 = __uint_as_float(__float_as_uint(p0) + (__float_as_uint(y0) << 23));
+    r1 = __uint_as_float(__float_as_uint(p1) + (__float_as_uint(y1) << 23));
 }
 
 // Two floats to packed bf16x2, round to nearest even; `lo` lands in bits 0-15.

@@ -84,6 +84,12 @@ __device__ __forceinline__ int unit_lower_bound(const Units& t, int sc)
     return lo;
 }
 
+// The unit that contains sub-chunk sc (units tile the sub-chunks in order).
+__device__ __forceinline__ int unit_of_subchunk(const Units& t, int sc)
+{
+    return unit_lower_bound(t, sc + 1) - 1;
+}
+
 __device__ __forceinline__ void unit_range(const Units& t, int u, int* anchor, int64_t* s,
                                            int64_t* e)
 {
