@@ -49,6 +49,9 @@ def parse_args():
                     help="skip timing the per-sub-chunk selection mode alongside")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle sample")
+    ap.add_argument("--sweep", action="store_true",
+                    help="clustering-threshold sweep (theta x L_max) on planted-topic data: cluster sizes, "
+                         "overlap ratio rho, boundary recall and step time (one JSON line)")
     return ap.parse_args()
 
 
@@ -401,6 +404,147 @@ def run_scale(args):
     return 0
 
 
+SWEEP_WORKLOAD = "llama8b-128k-topics"
+SWEEP_THETAS = (0.95, 0.97, 0.99)
+SWEEP_SMAX = (2, 4, 8)
+
+
+def cosine_stats(fp: np.ndarray) -> dict:
+    """Distribution of cos(v_i, v_{i+1}) over consecutive sub-chunks (the paper's Table 1 format)."""
+    vt = fp / np.linalg.norm(fp, axis=1, keepdims=True)
+    c = np.sum(vt[1:] * vt[:-1], axis=1)
+    return {"mean": float(c.mean()), "min": float(c.min()), "max": float(c.max()),
+            "p10": float(np.percentile(c, 10)), "median": float(np.median(c)),
+            "p90": float(np.percentile(c, 90))}
+
+
+def boundary_recall(w, unit_start: np.ndarray) -> dict:
+    """Share of planted topic boundaries at which a cluster opens: at the
+    sub-chunk that contains the boundary or at the first one after it."""
+    from synth import topic_segments
+
+    starts, _ = topic_segments(w, 0, w.seed)
+    opened = set(int(x) for x in unit_start[:-1])
+    hits = 0
+    for b in starts[1:]:
+        i = int(b) // w.sub_chunk
+        hits += (i in opened) or (i + 1 in opened)
+    return {"boundaries": int(len(starts) - 1), "recalled": int(hits)}
+
+
+def run_sweep(args):
+    """Alg. 1's threshold branch on planted-topic data: for every (L_max, theta),
+    the step time, the clusters formed, their retrieval calls, and the overlap
+    ratio of Sec. IV-C against the per-sub-chunk union (both with member
+    queries scored on the cluster's candidates and with the members' own
+    per-sub-chunk selections)."""
+    import torch
+
+    import paper_2609_31568_gb300 as pkg
+    from paper_2609_31568_gb300 import fidelity as F
+    from paper_2609_31568_gb300 import scale as S
+
+    pkg.build()
+    S.load()
+    w0 = workload(args.workload if args.workload != DEFAULT_WORKLOAD else SWEEP_WORKLOAD)
+    q, k, v = generate_layer(w0)
+    dev = [torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)]
+    stream = torch.cuda.current_stream()
+    CL, SUB = S.SCALE_MODE_PER_CLUSTER, S.SCALE_MODE_PER_SUBCHUNK
+    peaks = load_peaks()
+
+    def step(p, mode, buf, steps, warmup):
+        for _ in range(warmup):
+            pkg.run_path(p, mode, *dev, buf)
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
+        torch.cuda.synchronize()
+        for e in ev:
+            e[0].record(stream)
+            S.scale_build_reps(p, dev[0], dev[1], buf.reps, buf.fingerprints, buf.unit_start,
+                               buf.n_units, buf.ws, stream)
+            e[1].record(stream)
+            S.scale_select(p, mode, 0, w0.n_tokens, buf.reps, buf.fingerprints, buf.unit_start,
+                           buf.n_units, buf.sel_blocks, buf.sel_count, None, buf.ws, stream)
+            e[2].record(stream)
+            S.scale_sparse_prefill(p, mode, 0, w0.n_tokens, *dev, buf.unit_start, buf.n_units,
+                                   buf.sel_blocks, buf.sel_count, buf.out, buf.ws, stream)
+            e[3].record(stream)
+        torch.cuda.synchronize()
+        st = S.scale_get_device_status(buf.ws)
+        if st != S.SCALE_OK:
+            raise RuntimeError(f"device status {st}: {S.status_string(st)}")
+        stages = [statistics.mean(x[j].elapsed_time(x[j + 1]) for x in ev) for j in range(3)]
+        return sum(stages), stages
+
+    steps, warmup = max(3, args.steps // 4), max(2, args.warmup)
+    pb = S.params_for(w0)
+    bufb = pkg.allocate(pb, SUB)
+    ms_b, st_b = step(pb, SUB, bufb, steps, warmup)
+    M = w0.n_subchunks
+    sel_sub = bufb.sel_blocks.cpu().numpy()
+    cnt_sub = bufb.sel_count.cpu().numpy()
+    _, calls_b = S.scale_retrieval_calls(pb, SUB, None, M)
+    keys_b = key_counts(w0, None, M, sel_sub, cnt_sub, True)
+    cos = cosine_stats(bufb.fingerprints.double().cpu().numpy())
+    del bufb
+
+    rows = []
+    for s_max in SWEEP_SMAX:
+        for theta in SWEEP_THETAS:
+            w = w0.replace(max_cluster_subchunks=s_max, theta=theta)
+            p = S.params_for(w)
+            buf = pkg.allocate(p, CL)
+            ms, st = step(p, CL, buf, steps, warmup)
+            n = int(buf.n_units.item())
+            us = buf.unit_start[: n + 1].cpu().numpy()
+            sizes = np.diff(us)
+            sel = buf.sel_blocks.cpu().numpy()
+            cnt = buf.sel_count.cpu().numpy()
+            same = {}
+            for j in range(1, s_max):
+                fpj = F.member_query_fingerprints(buf.fingerprints, buf.unit_start, n, j)
+                sj, cj = torch.empty_like(buf.sel_blocks), torch.empty_like(buf.sel_count)
+                S.scale_select(p, CL, 0, w.n_tokens, buf.reps, fpj, buf.unit_start, buf.n_units,
+                               sj, cj, None, buf.ws, stream)
+                same[j] = (sj.cpu().numpy(), cj.cpu().numpy())
+            if S.scale_get_device_status(buf.ws) != S.SCALE_OK:
+                raise RuntimeError("device status after member selections")
+            rho_same, _ = F.overlap_ratios(us, sel, cnt, lambda u, j: same[j][0][u, : same[j][1][u]])
+            rho_own, _ = F.overlap_ratios(
+                us, sel, cnt, lambda u, j: sel_sub[us[u] + j, : cnt_sub[us[u] + j]])
+            _, calls = S.scale_retrieval_calls(p, CL, us, n)
+            keys = key_counts(w, us, n, sel, cnt, False)
+            flops = 4.0 * w.head_dim * w.num_q_heads * keys
+            hist = {str(c): int(np.count_nonzero(sizes == c)) for c in range(1, s_max + 1)}
+            rows.append({
+                "l_max_subchunks": s_max, "theta": theta, "ms_per_step": ms,
+                "stages_ms": {"build_reps": st[0], "select": st[1], "sparse_attention": st[2]},
+                "units": n, "retrieval_calls": calls,
+                "mean_cluster_tokens": float(w.n_tokens / n), "cluster_sizes": hist,
+                "full_clusters": float(np.mean(sizes == s_max)),
+                "rho_same_candidates": F.summary(rho_same), "rho_own_selection": F.summary(rho_own),
+                "boundary_recall": boundary_recall(w, us),
+                "attn_tflops": flops / (st[2] / 1e3) / 1e12,
+                "attn_flops_vs_per_subchunk": keys / keys_b,
+            })
+            del buf
+            torch.cuda.empty_cache()
+    line = {
+        "metric": "clustering-threshold sweep: cluster sizes, overlap ratio, retrieval calls, step time",
+        "workload": w0.name, "n_tokens": w0.n_tokens, "sub_chunk": w0.sub_chunk,
+        "outer_chunk": w0.outer_chunk, "block_size": w0.block_size, "top_k_blocks": w0.top_k,
+        "top_k_tokens": w0.top_k * w0.block_size, "steps": steps, "warmup": warmup,
+        "data": "synthetic, planted topics", "consecutive_cosine": cos,
+        "per_subchunk": {"ms_per_step": ms_b, "retrieval_calls": calls_b, "units": M,
+                         "stages_ms": {"build_reps": st_b[0], "select": st_b[1], "sparse_attention": st_b[2]},
+                         "attn_tflops": 4.0 * w0.head_dim * w0.num_q_heads * keys_b / (st_b[2] / 1e3) / 1e12},
+        "peak_bf16_sustained_tflops": peaks["bf16_sustained"],
+        "sweep": rows,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_stack(args):
     """Multi-layer workload: attention-only TTFT of a chunked prefill over all layers.
 
@@ -528,6 +672,8 @@ def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.sweep:
+        return run_sweep(args)
     if workload(args.workload).layers > 1:
         return run_stack(args)
     return run_scale(args)

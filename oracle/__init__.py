@@ -194,3 +194,33 @@ def run_path(w, q: np.ndarray, k: np.ndarray, v: np.ndarray, *, per_subchunk: bo
                                      per_subchunk=per_subchunk, unit_start=us, sel=s["sel"],
                                      sel_count=s["sel_count"], rows=out["rows"])
     return out
+
+
+def member_selection(w, reps: np.ndarray, v: np.ndarray, unit_start: np.ndarray, j: int,
+                     select_scale: float = 1.0):
+    """Selection of every cluster scored with its member j's fingerprint in place
+    of the anchor's, against the cluster's own candidate blocks (Sec. IV-C's
+    per-sub-chunk retrieval "against the same KV cache"); units with at most j
+    sub-chunks keep their anchor."""
+    v2 = np.array(v, np.float64, copy=True)
+    for u in range(len(unit_start) - 1):
+        a, b = int(unit_start[u]), int(unit_start[u + 1])
+        if b - a > j:
+            v2[a] = v[a + j]
+    return select(num_q_heads=w.num_q_heads, n_tokens=w.n_tokens, sub_chunk=w.sub_chunk,
+                  block_size=w.block_size, top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                  select_scale=select_scale, per_subchunk=False, reps=reps, v=v2,
+                  unit_start=unit_start)
+
+
+def overlap_ratio(anchor_blocks, member_blocks) -> float:
+    """Overlap ratio of one cluster (Sec. IV-C): the share of the anchor's
+    selected blocks that at least one other member would also select.
+    anchor_blocks: the anchor's selection; member_blocks: one selection per
+    other member."""
+    anchor = {int(b) for b in anchor_blocks}
+    others = set()
+    for m in member_blocks:
+        others |= {int(b) for b in m}
+    return len(anchor & others) / len(anchor)
+

@@ -4,7 +4,7 @@
 ``_build.build()`` compiles it in-tree with nvcc.
 """
 
-from . import scale  # noqa: F401
+from . import fidelity, scale  # noqa: F401
 from ._build import build  # noqa: F401
 from .scale import (  # noqa: F401
     SCALE_MODE_PER_CLUSTER,

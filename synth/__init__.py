@@ -12,5 +12,6 @@ from .generate import (  # noqa: F401
     bf16_bits_to_f32,
     f64_to_bf16_bits,
     generate_layer,
+    topic_segments,
     workload,
 )

@@ -11,6 +11,24 @@ in for them. The recipe, per layer:
    in the order drawn, plus N(0, 1) noise per element;
 3. queries: a component id per (token, query head) from the centroid set of
    the query head's KV head (``h // (H_q / H_kv)``), plus N(0, 1) noise;
+   With planted topics (``topics`` > 0) the sequence is cut into segments of
+   exponentially distributed length (mean ``topic_len`` tokens, boundaries
+   at any token), each segment carries one of ``topics`` topics (never the
+   same as the segment before), each topic owns a contiguous group of
+   ``components / topics`` components, and every key and query of a segment
+   draws its component id from that group only. On top of the mixture,
+   every query head carries a fixed shared direction of norm
+   ``shared_norm`` and every segment adds its topic's direction of norm
+   ``topic_norm`` (one per topic and KV head, on the queries of that KV
+   head's group and on its keys); both live in the lowest-frequency quarter
+   of the rotary pairs, as the large low-frequency query components of
+   trained models do, so sub-chunk fingerprints stay close within a topic,
+   drift slowly with distance (the slow rotation of those pairs), and jump
+   at a boundary. A drift in the same band, shared by all query heads, a stationary
+   AR(1) process over knots 1024 tokens apart (stationary norm
+   ``wobble_norm``, correlation ``wobble_corr`` from one knot to the next,
+   linear between knots, moving in ``wobble_dims`` fixed random directions
+   of the band), spreads the similarity of consecutive sub-chunks;
 4. values: N(0, 1);
 5. optional rotate-half RoPE at absolute positions ``0..N-1`` on Q and K;
 6. mixing, noise and RoPE are computed in float32 (the centroids in
@@ -51,6 +69,13 @@ class Workload:
     layers: int = 1
     seed: int = 0
     theta: float = -1.0
+    topics: int = 0          # planted topics (0: none)
+    topic_len: int = 0       # mean topic segment length in tokens
+    topic_norm: float = 0.0  # norm of a topic's low-frequency direction
+    shared_norm: float = 0.0  # norm of each query head's shared low-frequency direction
+    wobble_norm: float = 0.0  # stationary norm of the low-frequency drift (all query heads)
+    wobble_corr: float = 0.0  # its correlation from one 1024-token knot to the next
+    wobble_dims: int = 0      # directions the drift moves in (0: the whole band)
 
     def replace(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
@@ -84,6 +109,14 @@ WORKLOADS: dict[str, Workload] = {
     "llama8b-1m": Workload("llama8b-1m", 32, 8, 128, 1048576, 4096, 16, 65536, 256, 128, 128, 1024,
                            1024, 500000.0, False),
 }
+
+
+# Planted-topic variant for the clustering-threshold sweep: the paper's sub-chunk
+# L = 512 and outer chunk 8192, k = 64 blocks of 128 = 8192 tokens, 128K context.
+WORKLOADS["llama8b-128k-topics"] = Workload(
+    "llama8b-128k-topics", 32, 8, 128, 131072, 512, 8, 8192, 128, 64, 128, 512, 256, 500000.0, False,
+    theta=0.95, topics=16, topic_len=16384, topic_norm=3.0, shared_norm=6.0, wobble_norm=4.0,
+    wobble_corr=0.96, wobble_dims=2)
 
 
 def workload(name: str, **overrides) -> Workload:
@@ -137,6 +170,71 @@ def _rope(x: np.ndarray, pos: np.ndarray, base: float) -> np.ndarray:
     return np.concatenate([lo * c - hi * s, hi * c + lo * s], axis=-1)
 
 
+def topic_segments(w: Workload, layer: int, seed: int):
+    """(segment start tokens, topic of each segment) for planted topics."""
+    rng = np.random.default_rng([seed, layer, 4])
+    starts, topics = [0], [int(rng.integers(0, w.topics))]
+    while True:
+        nxt = starts[-1] + 1 + int(rng.exponential(w.topic_len))
+        if nxt >= w.n_tokens:
+            break
+        t = int(rng.integers(0, w.topics - 1))
+        starts.append(nxt)
+        topics.append(t if t < topics[-1] else t + 1)  # a different topic
+    return np.array(starts, np.int64), np.array(topics, np.int64)
+
+
+def _low_band(w: Workload) -> np.ndarray:
+    """Dims of the lowest-frequency quarter of the rotate-half rotary pairs."""
+    half = w.head_dim // 2
+    pairs = np.arange(half - half // 4, half)
+    return np.concatenate([pairs, pairs + half])
+
+
+def _topic_dirs(w: Workload, layer: int, seed: int):
+    """(shared [H_q, d_h], topic [topics, H_kv, d_h]) low-frequency directions."""
+    rng = np.random.default_rng([seed, layer, 5])
+    band = _low_band(w)
+    shared = np.zeros((w.num_q_heads, w.head_dim))
+    shared[:, band] = _unit_rows(rng.standard_normal((w.num_q_heads, band.size))) * w.shared_norm
+    topic = np.zeros((w.topics, w.num_kv_heads, w.head_dim))
+    topic[:, :, band] = _unit_rows(rng.standard_normal((w.topics, w.num_kv_heads, band.size))) * w.topic_norm
+    return shared.astype(np.float32), topic.astype(np.float32)
+
+
+WOBBLE_KNOT = 1024
+
+
+def _wobble(w: Workload, layer: int, seed: int, pos: np.ndarray) -> np.ndarray:
+    """Low-frequency drift [T, 1, d_h] (the same for every query head) at positions pos."""
+    rng = np.random.default_rng([seed, layer, 6])
+    band = _low_band(w)
+    r = w.wobble_dims or band.size
+    basis = np.linalg.qr(rng.standard_normal((band.size, r)))[0]  # orthonormal columns
+    n_knots = w.n_tokens // WOBBLE_KNOT + 2
+    sd = w.wobble_norm / np.sqrt(r)
+    a = w.wobble_corr
+    z = rng.standard_normal((n_knots, 1, r))
+    knots = np.empty_like(z)
+    knots[0] = sd * z[0]
+    for j in range(1, n_knots):
+        knots[j] = a * knots[j - 1] + np.sqrt(1.0 - a * a) * sd * z[j]
+    j = pos // WOBBLE_KNOT
+    f = ((pos % WOBBLE_KNOT) / WOBBLE_KNOT)[:, None, None]
+    out = np.zeros((pos.size, 1, w.head_dim), np.float32)
+    out[:, :, band] = (((1.0 - f) * knots[j] + f * knots[j + 1]) @ basis.T).astype(np.float32)
+    return out
+
+
+def _component_ids(w: Workload, rng, shape, pos, segs):
+    if not w.topics:
+        return rng.integers(0, w.components, size=shape)
+    group = w.components // w.topics
+    starts, topics = segs
+    topic = topics[np.searchsorted(starts, pos, side="right") - 1]
+    return topic[:, None] * group + rng.integers(0, group, size=shape)
+
+
 def _chunk(w: Workload, layer: int, seed: int, cents, ch: int):
     t0 = ch * CHUNK
     t1 = min(w.n_tokens, t0 + CHUNK)
@@ -145,13 +243,23 @@ def _chunk(w: Workload, layer: int, seed: int, cents, ch: int):
     kvh = np.arange(w.num_kv_heads)
     qkv = np.arange(w.num_q_heads) // w.group
 
+    segs = topic_segments(w, layer, seed) if w.topics else None
     rk = np.random.default_rng([seed, layer, 1, ch])
-    kid = rk.integers(0, w.components, size=(T, w.num_kv_heads))
+    kid = _component_ids(w, rk, (T, w.num_kv_heads), pos, segs)
     k = _mix(w, cents, kvh, kid, pos) + rk.standard_normal((T, w.num_kv_heads, w.head_dim), dtype=np.float32)
 
     rq = np.random.default_rng([seed, layer, 2, ch])
-    qid = rq.integers(0, w.components, size=(T, w.num_q_heads))
+    qid = _component_ids(w, rq, (T, w.num_q_heads), pos, segs)
     q = _mix(w, cents, qkv, qid, pos) + rq.standard_normal((T, w.num_q_heads, w.head_dim), dtype=np.float32)
+
+    if w.topics:
+        shared, topic = _topic_dirs(w, layer, seed)
+        starts, tops = segs
+        tp = tops[np.searchsorted(starts, pos, side="right") - 1]
+        k = k + topic[tp]
+        q = q + shared[None] + topic[tp][:, qkv]
+        if w.wobble_norm:
+            q = q + _wobble(w, layer, seed, pos)
 
     rv = np.random.default_rng([seed, layer, 3, ch])
     v = rv.standard_normal((T, w.num_kv_heads, w.head_dim), dtype=np.float32)

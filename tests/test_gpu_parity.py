@@ -229,6 +229,54 @@ def test_end_to_end_parity_sampled(name, n_random, mode):
     assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
 
 
+# --------------------------------------------------------------------------- threshold sweep
+
+
+@pytest.mark.parametrize("s_max,theta", [(4, 0.97), (8, 0.95), (8, 0.99)])
+def test_planted_topic_sweep_parity(s_max, theta):
+    """Alg. 1 with a real threshold on planted-topic data (32K tokens, L = 512):
+    the GPU's clusters, the anchors' selections, every member's selection
+    against the cluster's candidates, and the overlap ratio of Sec. IV-C match
+    the oracle."""
+    from paper_2609_31568_gb300 import fidelity as F
+
+    w, q, k, v, dev = inputs("llama8b-128k-topics", n_tokens=32768, max_cluster_subchunks=s_max,
+                             theta=theta)
+    p, buf = gpu_path(w, PER_CLUSTER, dev)
+    ref = oracle_path(w, q, k, v, PER_CLUSTER)
+    assert ref["margin"] > 1e-5  # every admission decision is far from theta in fp32 terms
+    n = int(buf.n_units.item())
+    us = buf.unit_start[: n + 1].cpu().numpy()
+    assert us.tolist() == ref["unit_start"].tolist()
+    assert 1 < n < w.n_subchunks
+    sel = buf.sel_blocks.cpu().numpy()[:n, : w.top_k]
+    cnt = buf.sel_count.cpu().numpy()[:n]
+    same, _ = compare_selection(sel, cnt, ref)
+    gpu_m, ref_m = {}, {}
+    for j in range(1, s_max):
+        fpj = F.member_query_fingerprints(buf.fingerprints, buf.unit_start, n, j)
+        sj, cj = torch.empty_like(buf.sel_blocks), torch.empty_like(buf.sel_count)
+        S.scale_select(p, PER_CLUSTER, 0, w.n_tokens, buf.reps, fpj, buf.unit_start, buf.n_units,
+                       sj, cj, None, buf.ws)
+        torch.cuda.synchronize()
+        assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
+        r = oracle.member_selection(w, ref["reps"], ref["fingerprints"], ref["unit_start"], j)
+        gpu_m[j] = (sj.cpu().numpy()[:n, : w.top_k], cj.cpu().numpy()[:n])
+        ref_m[j] = r
+        ok_j, _ = compare_selection(*gpu_m[j], r)
+        same &= ok_j
+    rho, units = F.overlap_ratios(us, sel, cnt, lambda u, j: gpu_m[j][0][u, : gpu_m[j][1][u]])
+    sizes = np.diff(ref["unit_start"])
+    for r_gpu, u in zip(rho, units):
+        if not same[u]:
+            continue  # a near-tie changed one of the selections involved
+        want = oracle.overlap_ratio(ref["sel"][u, : ref["sel_count"][u]],
+                                    [ref_m[j]["sel"][u, : ref_m[j]["sel_count"][u]] for j in range(1, sizes[u])])
+        assert r_gpu == want
+    assert len(units) == int(np.count_nonzero((sizes >= 2) & (ref["sel_count"] > 0)))
+    print(f"L_max={s_max}L theta={theta}: {n} units, rho min {rho.min():.3f} median {np.median(rho):.3f}")
+
+
 # --------------------------------------------------------------------------- invariants
 
 
