@@ -68,6 +68,18 @@ def load_peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
 
 
+def launches(w, selects: int = 1) -> dict:
+    """Kernels each call of the path launches for workload w (block size 1
+    skips the representatives, scores in four kernels and gathers the distant
+    keys through a per-unit list)."""
+    tok = w.block_size == 1
+    build = (3 if tok else 4) + (1 if w.max_cluster_subchunks > 1 else 0)
+    select = 5 if tok else 4
+    attend = 2 if tok else 1
+    return {"build_reps": build, "select": select * selects, "attend": attend * selects,
+            "total": build + (select + attend) * selects}
+
+
 def key_counts(w, unit_start, n_units, sel, cnt, per_subchunk):
     """Sum over query rows of |K(p)|, the distinct keys each row attends to (Eq. 10)."""
     total = 0
@@ -287,8 +299,7 @@ def run_scale(args):
             S.scale_build_reps(p, dev[0], dev[1], buf_.reps, buf_.fingerprints, buf_.unit_start,
                                buf_.n_units, buf_.ws, stream)
             e[1].record(stream)
-            S.scale_select(p, mode_, 0, w.n_tokens, buf_.reps, buf_.fingerprints, buf_.unit_start,
-                           buf_.n_units, buf_.sel_blocks, buf_.sel_count, None, buf_.ws, stream)
+            S.select(p, mode_, 0, w.n_tokens, dev[1], buf_, stream)
             e[2].record(stream)
             S.scale_sparse_prefill(p, mode_, 0, w.n_tokens, *dev, buf_.unit_start, buf_.n_units,
                                    buf_.sel_blocks, buf_.sel_count, buf_.out, buf_.ws, stream)
@@ -350,7 +361,7 @@ def run_scale(args):
                      "frac_of_burst": achieved / peaks["bf16"],
                      "peak_source": f"bf16 sustained, of {peaks['source']}",
                      "algorithmic_flops_per_launch": flops, "traffic": profile_traffic()},
-        "gpu_launches": args.steps * (10 if w.max_cluster_subchunks > 1 else 9),
+        "gpu_launches": args.steps * launches(w)["total"],
         "clocks": clk,
     }
 
@@ -463,8 +474,7 @@ def run_sweep(args):
             S.scale_build_reps(p, dev[0], dev[1], buf.reps, buf.fingerprints, buf.unit_start,
                                buf.n_units, buf.ws, stream)
             e[1].record(stream)
-            S.scale_select(p, mode, 0, w0.n_tokens, buf.reps, buf.fingerprints, buf.unit_start,
-                           buf.n_units, buf.sel_blocks, buf.sel_count, None, buf.ws, stream)
+            S.select(p, mode, 0, w0.n_tokens, dev[1], buf, stream)
             e[2].record(stream)
             S.scale_sparse_prefill(p, mode, 0, w0.n_tokens, *dev, buf.unit_start, buf.n_units,
                                    buf.sel_blocks, buf.sel_count, buf.out, buf.ws, stream)
@@ -584,8 +594,7 @@ def run_stack(args):
             i = 0
             for t0, t1 in chunks:
                 for dev, b in zip(layers, bufs):
-                    S.scale_select(p, mode, t0, t1, b.reps, b.fingerprints, b.unit_start, b.n_units,
-                                   b.sel_blocks, b.sel_count, None, b.ws, stream)
+                    S.select(p, mode, t0, t1, dev[1], b, stream)
                     if ev is not None:
                         ev[i][0].record(stream)
                     S.scale_sparse_prefill(p, mode, t0, t1, *dev, b.unit_start, b.n_units, b.sel_blocks,
@@ -651,7 +660,7 @@ def run_stack(args):
                      "frac": achieved / peaks["bf16_sustained"], "frac_of_burst": achieved / peaks["bf16"],
                      "peak_source": f"bf16 sustained, of {peaks['source']}",
                      "algorithmic_flops_per_step": flops, "traffic": None},
-        "gpu_launches": args.steps * w.layers * (5 + len(chunks) * 5),
+        "gpu_launches": args.steps * w.layers * launches(w, len(chunks))["total"],
         "clocks": clk,
     }
     if not args.no_baseline_mode and rank == 0:

@@ -112,7 +112,7 @@ int scale_workspace_init(void *ws, size_t ws_bytes, scale_stream_t stream);
  * outer_chunk tokens, producing unit_start[0..n_units] (entries after
  * n_units are set to M) and *n_units (device).
  *   q            bf16 [N][H_q][128]        k  bf16 [N][H_kv][128]
- *   reps         fp32 [H_kv][nb][128]      out
+ *   reps         fp32 [H_kv][nb][128]      out (may be NULL when block_size is 1)
  *   fingerprints fp32 [M][H_q*128]         out (raw means v_i, not normalised)
  *   unit_start   int32 [M+1]               out
  *   n_units      int32 [1]                 out (device)
@@ -160,6 +160,28 @@ int scale_select(const scale_params_t *p, int32_t mode, int64_t tok_begin, int64
                  const int32_t *n_units, int32_t *sel_blocks, int32_t *sel_count,
                  float *sel_scores, void *ws, size_t ws_bytes, scale_stream_t stream);
 
+/* Steps (b) and (c) at token granularity (block_size must be 1): the rule of
+ * scale_select with every key as its own block, which is the paper's own
+ * selection (Sec. V-A3, Eq. 9, TokenSelect's head soft-voting over tokens):
+ *   z_{h,t} = select_scale * v_a^(h) . k_t^(h / g)  for n_sink <= t < W_u,
+ *   p_h = softmax_t(z_h), score_t = sum_h p_{h,t}, top_k tokens (ties to the
+ *   lower index), ascending.
+ * The scores are computed from K directly on the tensor cores (the fp32
+ * fingerprint split into three bf16 parts, fp32 accumulation), so
+ * scale_build_reps may be given reps = NULL for block size 1.
+ *   k           bf16 [N][H_kv][128]
+ *   sel_tokens  int32 [M][top_k] out (ascending token indices, -1 padded)
+ *   sel_count   int32 [M] out
+ *   sel_scores  fp32 [M][N] or NULL: score_t on the candidates, NaN elsewhere.
+ * Same range rule, modes and workspace as scale_select. H_q / H_kv must be 1,
+ * 2, 4 or 8 (SCALE_ERR_UNSUPPORTED otherwise); block_size != 1 gives
+ * SCALE_ERR_INVALID_ARG (and scale_select gives SCALE_ERR_UNSUPPORTED for
+ * block size 1). */
+int scale_select_tokens(const scale_params_t *p, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                        const void *k, const float *fingerprints, const int32_t *unit_start,
+                        const int32_t *n_units, int32_t *sel_tokens, int32_t *sel_count,
+                        float *sel_scores, void *ws, size_t ws_bytes, scale_stream_t stream);
+
 /* Step (d). Eq. 10 for every query row p of every unit u starting in
  * [tok_begin, tok_end) and every query head h:
  *   keys K(p) = ([0, n_sink) U selected blocks of u U [W_u, e_u)) n [0, p],
@@ -171,7 +193,10 @@ int scale_select(const scale_params_t *p, int32_t mode, int64_t tok_begin, int64
  * not written. Same range rule as scale_select.
  *   q, out bf16 [N][H_q][128];  k, v bf16 [N][H_kv][128];
  *   sel_blocks / sel_count as written by scale_select (any selection obeying
- *   the same layout is accepted; entries outside [0, nb) are ignored). */
+ *   the same layout is accepted; entries outside [0, nb) are ignored). With
+ *   block_size 1 they are scale_select_tokens' token lists, and the kernel
+ *   gathers the selected keys and values row by row (entries outside
+ *   [n_sink, W_u) or not above their predecessor are ignored). */
 int scale_sparse_prefill(const scale_params_t *p, int32_t mode, int64_t tok_begin,
                          int64_t tok_end, const void *q, const void *k, const void *v,
                          const int32_t *unit_start, const int32_t *n_units,

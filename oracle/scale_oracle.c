@@ -244,57 +244,66 @@ int oracle_select(int Hq, int Hkv, int dh, int64_t N, int L, int B, int k, int n
     const int g = Hq / Hkv;
     const int64_t nb = (N + B - 1) / B;
     const int64_t D = (int64_t)Hq * dh;
-    scored_t *cand = (scored_t *)malloc(sizeof(scored_t) * (size_t)nb);
-    double *z = (double *)malloc(sizeof(double) * (size_t)nb);
-    double *score = (double *)malloc(sizeof(double) * (size_t)nb);
-    if (!cand || !z || !score) {
-        free(cand); free(z); free(score);
-        return -1;
-    }
-    for (int64_t u = 0; u < n_units; ++u) {
-        int64_t a, s, e;
-        unit_range(per_subchunk, unit_start, u, L, N, &a, &s, &e);
-        const int64_t W = (s - n_local > 0) ? s - n_local : 0;
-
-        /* R4: candidate blocks have a token in [n_sink, W). */
-        int64_t nc = 0;
-        for (int64_t b = 0; b < nb; ++b) {
-            score[b] = NAN;
-            if (b * B < W && (b + 1) * B > n_sink) cand[nc++].b = (int32_t)b;
+    int err = 0;
+    /* Units are independent; each thread takes whole units with its own
+     * scratch, so the arithmetic of a unit is the same as in a serial loop. */
+#pragma omp parallel
+    {
+        scored_t *cand = (scored_t *)malloc(sizeof(scored_t) * (size_t)nb);
+        double *z = (double *)malloc(sizeof(double) * (size_t)nb);
+        double *score = (double *)malloc(sizeof(double) * (size_t)nb);
+        const int ok = cand && z && score;
+        if (!ok) {
+#pragma omp atomic write
+            err = 1;
         }
-        for (int64_t i = 0; i < nc; ++i) score[cand[i].b] = 0.0;
+#pragma omp for schedule(dynamic, 1)
+        for (int64_t u = 0; u < n_units; ++u) {
+            if (!ok) continue;
+            int64_t a, s, e;
+            unit_range(per_subchunk, unit_start, u, L, N, &a, &s, &e);
+            const int64_t W = (s - n_local > 0) ? s - n_local : 0;
 
-        for (int h = 0; h < Hq && nc > 0; ++h) {
-            const double *vh = v + a * D + (int64_t)h * dh;
-            const double *rj = reps + (int64_t)(h / g) * nb * dh;
-            double zmax = -INFINITY;
-            for (int64_t i = 0; i < nc; ++i) {
-                const double *r = rj + (int64_t)cand[i].b * dh;
-                double dot = 0.0;
-                for (int d = 0; d < dh; ++d) dot += vh[d] * r[d];
-                z[i] = sigma * dot;
-                if (z[i] > zmax) zmax = z[i];
+            /* R4: candidate blocks have a token in [n_sink, W). */
+            int64_t nc = 0;
+            for (int64_t b = 0; b < nb; ++b) {
+                score[b] = NAN;
+                if (b * B < W && (b + 1) * B > n_sink) cand[nc++].b = (int32_t)b;
             }
-            double den = 0.0;
-            for (int64_t i = 0; i < nc; ++i) den += exp(z[i] - zmax);
-            for (int64_t i = 0; i < nc; ++i) score[cand[i].b] += exp(z[i] - zmax) / den;
-        }
+            for (int64_t i = 0; i < nc; ++i) score[cand[i].b] = 0.0;
 
-        for (int64_t i = 0; i < nc; ++i) cand[i].score = score[cand[i].b];
-        qsort(cand, (size_t)nc, sizeof(scored_t), cmp_scored);
-        const int64_t take = nc < k ? nc : k;
-        int32_t *su = sel + u * (int64_t)k;
-        for (int64_t i = 0; i < k; ++i) su[i] = -1;
-        for (int64_t i = 0; i < take; ++i) su[i] = cand[i].b;
-        qsort(su, (size_t)take, sizeof(int32_t), cmp_i32);
-        sel_count[u] = (int32_t)take;
-        cand_count[u] = (int32_t)nc;
-        gap[u] = (nc > k && k > 0) ? (cand[k - 1].score - cand[k].score) / cand[k - 1].score : INFINITY;
-        if (scores)
-            for (int64_t b = 0; b < nb; ++b) scores[u * nb + b] = score[b];
+            for (int h = 0; h < Hq && nc > 0; ++h) {
+                const double *vh = v + a * D + (int64_t)h * dh;
+                const double *rj = reps + (int64_t)(h / g) * nb * dh;
+                double zmax = -INFINITY;
+                for (int64_t i = 0; i < nc; ++i) {
+                    const double *r = rj + (int64_t)cand[i].b * dh;
+                    double dot = 0.0;
+                    for (int d = 0; d < dh; ++d) dot += vh[d] * r[d];
+                    z[i] = sigma * dot;
+                    if (z[i] > zmax) zmax = z[i];
+                }
+                double den = 0.0;
+                for (int64_t i = 0; i < nc; ++i) den += exp(z[i] - zmax);
+                for (int64_t i = 0; i < nc; ++i) score[cand[i].b] += exp(z[i] - zmax) / den;
+            }
+
+            for (int64_t i = 0; i < nc; ++i) cand[i].score = score[cand[i].b];
+            qsort(cand, (size_t)nc, sizeof(scored_t), cmp_scored);
+            const int64_t take = nc < k ? nc : k;
+            int32_t *su = sel + u * (int64_t)k;
+            for (int64_t i = 0; i < k; ++i) su[i] = -1;
+            for (int64_t i = 0; i < take; ++i) su[i] = cand[i].b;
+            qsort(su, (size_t)take, sizeof(int32_t), cmp_i32);
+            sel_count[u] = (int32_t)take;
+            cand_count[u] = (int32_t)nc;
+            gap[u] = (nc > k && k > 0) ? (cand[k - 1].score - cand[k].score) / cand[k - 1].score : INFINITY;
+            if (scores)
+                for (int64_t b = 0; b < nb; ++b) scores[u * nb + b] = score[b];
+        }
+        free(cand); free(z); free(score);
     }
-    free(cand); free(z); free(score);
-    return 0;
+    return err ? -1 : 0;
 }
 
 /* ---------------------------------------------------------------------------

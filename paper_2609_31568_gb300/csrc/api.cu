@@ -65,7 +65,13 @@ WsLayout ws_layout(const Derived& d)
     w.norms = take(static_cast<size_t>(d.M) * sizeof(float));
     w.gram = take(static_cast<size_t>(d.M) * d.S_max * sizeof(float));
     w.anchor = take(static_cast<size_t>(d.M) * sizeof(int32_t));
-    w.logits = take(static_cast<size_t>(d.M) * d.Hq * d.nb * sizeof(float));
+    const bool tok = d.B == 1;
+    w.logits = take(tok ? 0 : static_cast<size_t>(d.M) * d.Hq * d.nb * sizeof(float));
+    w.tok_split = take(tok ? static_cast<size_t>(3) * d.M * d.Hq * kHeadDim * 2 : 0);
+    const int64_t ranges = tok ? (d.N + tok_range(d) - 1) / tok_range(d) : 0;
+    w.tok_part = take(static_cast<size_t>(d.M) * d.Hq * ranges * 2 * sizeof(float));
+    w.tok_list = take(tok ? static_cast<size_t>(d.M) * (d.n_sink + d.k) * sizeof(int32_t) : 0);
+    w.tok_count = take(tok ? static_cast<size_t>(d.M) * sizeof(int32_t) : 0);
     w.stats = take(static_cast<size_t>(d.M) * d.Hq * 2 * sizeof(float));
     w.scores = take(static_cast<size_t>(d.M) * d.nb * sizeof(float));
     w.total = off;
@@ -125,7 +131,7 @@ Arena arena_layout(const Derived& d, int mode)
     a.k = take(static_cast<size_t>(d.N) * d.Hkv * kHeadDim * 2);
     a.v = take(static_cast<size_t>(d.N) * d.Hkv * kHeadDim * 2);
     a.out = take(static_cast<size_t>(d.N) * d.Hq * kHeadDim * 2);
-    a.reps = take(static_cast<size_t>(d.Hkv) * d.nb * kHeadDim * sizeof(float));
+    a.reps = take(d.B == 1 ? 0 : static_cast<size_t>(d.Hkv) * d.nb * kHeadDim * sizeof(float));
     a.fp = take(static_cast<size_t>(d.M) * d.D * sizeof(float));
     a.unit_start = take(static_cast<size_t>(d.M + 1) * sizeof(int32_t));
     a.n_units = take(sizeof(int32_t));
@@ -183,7 +189,7 @@ int scale_build_reps(const scale_params_t* p, const void* q, const void* k, floa
     Derived d;
     int rc = derive(p, &d);
     if (rc) return rc;
-    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(reps, 16) ||
+    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !(device_ptr(reps, 16) || (!reps && d.B == 1)) ||
         !device_ptr(fingerprints, 16) || !device_ptr(unit_start, 4) || !device_ptr(n_units, 4))
         return SCALE_ERR_INVALID_ARG;
     if ((rc = check_ws(d, ws, ws_bytes))) return rc;
@@ -200,6 +206,7 @@ int scale_select(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64
     int rc = derive(p, &d);
     if (rc) return rc;
     if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
+    if (d.B == 1) return SCALE_ERR_UNSUPPORTED;  // block size 1: scale_select_tokens
     if (!device_ptr(reps, 16) || !device_ptr(fingerprints, 16) || !device_ptr(sel_count, 4) ||
         (d.k > 0 && !device_ptr(sel_blocks, 4)) || (sel_scores && !device_ptr(sel_scores, 4)))
         return SCALE_ERR_INVALID_ARG;
@@ -210,6 +217,29 @@ int scale_select(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64
     return cuda_status(launch_select(d, mode, tok_begin, tok_end, reps, fingerprints, unit_start,
                                      n_units, sel_blocks, sel_count, sel_scores,
                                      static_cast<uint8_t*>(ws), stream));
+}
+
+int scale_select_tokens(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                        const void* k, const float* fingerprints, const int32_t* unit_start,
+                        const int32_t* n_units, int32_t* sel_tokens, int32_t* sel_count,
+                        float* sel_scores, void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (d.B != 1) return SCALE_ERR_INVALID_ARG;
+    if (d.g != 1 && d.g != 2 && d.g != 4 && d.g != 8) return SCALE_ERR_UNSUPPORTED;
+    if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
+    if (!device_ptr(k, 16) || !device_ptr(fingerprints, 16) || !device_ptr(sel_count, 4) ||
+        (d.k > 0 && !device_ptr(sel_tokens, 4)) || (sel_scores && !device_ptr(sel_scores, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if (mode == SCALE_MODE_PER_CLUSTER && (!device_ptr(unit_start, 4) || !device_ptr(n_units, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
+    if (tok_begin == tok_end) return SCALE_OK;
+    return cuda_status(launch_select_tokens(d, mode, tok_begin, tok_end, k, fingerprints, unit_start,
+                                            n_units, sel_tokens, sel_count, sel_scores,
+                                            static_cast<uint8_t*>(ws), g_timeout_ns.load(), stream));
 }
 
 int scale_sparse_prefill(const scale_params_t* p, int32_t mode, int64_t tok_begin,
@@ -223,7 +253,7 @@ int scale_sparse_prefill(const scale_params_t* p, int32_t mode, int64_t tok_begi
     if (rc) return rc;
     if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
     if (d.g % 2) return SCALE_ERR_UNSUPPORTED;
-    if (max_distant_segments(d) > kMaxSegments) return SCALE_ERR_UNSUPPORTED;
+    if (d.B > 1 && max_distant_segments(d) > kMaxSegments) return SCALE_ERR_UNSUPPORTED;
     if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(v, 16) || !device_ptr(out, 16) ||
         !device_ptr(sel_count, 4) || (d.k > 0 && !device_ptr(sel_blocks, 4)))
         return SCALE_ERR_INVALID_ARG;
@@ -308,7 +338,7 @@ int scale_prefill_host(const scale_params_t* p, int32_t mode, const void* q_host
     if (e != cudaSuccess) return SCALE_ERR_CUDA;
     void* ws = base + A.ws;
     const size_t wsb = arena_bytes - A.ws;
-    auto* reps = reinterpret_cast<float*>(base + A.reps);
+    auto* reps = d.B == 1 ? nullptr : reinterpret_cast<float*>(base + A.reps);
     auto* fp = reinterpret_cast<float*>(base + A.fp);
     auto* us = reinterpret_cast<int32_t*>(base + A.unit_start);
     auto* nu = reinterpret_cast<int32_t*>(base + A.n_units);
@@ -316,7 +346,9 @@ int scale_prefill_host(const scale_params_t* p, int32_t mode, const void* q_host
     auto* cnt = reinterpret_cast<int32_t*>(base + A.sel_count);
     if ((rc = scale_workspace_init(ws, wsb, stream))) return rc;
     if ((rc = scale_build_reps(p, base + A.q, base + A.k, reps, fp, us, nu, ws, wsb, stream))) return rc;
-    if ((rc = scale_select(p, mode, 0, d.N, reps, fp, us, nu, sel, cnt, nullptr, ws, wsb, stream))) return rc;
+    rc = d.B == 1 ? scale_select_tokens(p, mode, 0, d.N, base + A.k, fp, us, nu, sel, cnt, nullptr, ws, wsb, stream)
+                  : scale_select(p, mode, 0, d.N, reps, fp, us, nu, sel, cnt, nullptr, ws, wsb, stream);
+    if (rc) return rc;
     if ((rc = scale_sparse_prefill(p, mode, 0, d.N, base + A.q, base + A.k, base + A.v, us, nu, sel,
                                    cnt, base + A.out, ws, wsb, stream)))
         return rc;

@@ -66,7 +66,8 @@ extern "C" int scale_build_reps_noalloc(const scale_params_t* p, const void* q, 
     Derived d;
     int rc = derive(p, &d);
     if (rc) return rc;
-    if (!dev_ptr(q, 16) || !dev_ptr(k, 16) || !dev_ptr(reps, 16) || !dev_ptr(fingerprints, 16) ||
+    if (!dev_ptr(q, 16) || !dev_ptr(k, 16) || !(dev_ptr(reps, 16) || (!reps && d.B == 1)) ||
+        !dev_ptr(fingerprints, 16) ||
         !dev_ptr(unit_start, 4) || !dev_ptr(n_units, 4))
         return SCALE_ERR_INVALID_ARG;
     // Step (a) uses the workspace prefix that ends where the selection's regions begin.

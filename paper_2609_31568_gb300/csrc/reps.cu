@@ -240,8 +240,9 @@ cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, fl
     int32_t* flag = reinterpret_cast<int32_t*>(ws + lay.anchor);
 
     const int row_chunks = d.Hkv * (kHeadDim / 8);
-    k_block_reps<<<static_cast<unsigned>(d.nb), row_chunks, 0, st>>>(
-        static_cast<const uint4*>(k), d.N, row_chunks, d.B, d.nb, reps);
+    if (reps)  // block size 1 may skip them: token-level selection reads K itself
+        k_block_reps<<<static_cast<unsigned>(d.nb), row_chunks, 0, st>>>(
+            static_cast<const uint4*>(k), d.N, row_chunks, d.B, d.nb, reps);
 
     const int D8 = d.D / 8;
     const int split_len = (d.L + d.fp_splits - 1) / d.fp_splits;

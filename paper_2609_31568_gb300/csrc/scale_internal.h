@@ -43,7 +43,11 @@ struct WsLayout {
     size_t norms;       // fp32 [M]
     size_t gram;        // fp32 [M][S_max]   cosine of sub-chunk i with i+d
     size_t anchor;      // int32 [M]         1 if sub-chunk i opens a cluster
-    size_t logits;      // fp32 [M][H_q][nb]
+    size_t logits;      // fp32 [M][H_q][nb]     (block size > 1 only)
+    size_t tok_split;   // bf16 [3][H_kv][M][g][128]  fingerprint parts (block size 1 only)
+    size_t tok_part;    // float2 [M][H_q][ranges]    per-range softmax partials (block size 1 only)
+    size_t tok_list;    // int32 [M][n_sink + k]      distant token list per unit (block size 1 only)
+    size_t tok_count;   // int32 [M]                  its length
     size_t stats;       // fp32 [M][H_q][2]  (row max, 1 / row sum)
     size_t scores;      // fp32 [M][nb]
     size_t total;
@@ -126,6 +130,14 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
                                   const int32_t* sel_blocks, const int32_t* sel_count, void* out,
                                   uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 cudaError_t launch_wait_selftest(uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
+cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_end, const float* scores,
+                        int32_t* sel, int32_t* sel_count, cudaStream_t st);
+cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
+                                 const void* k, const float* fingerprints, const int32_t* unit_start,
+                                 const int32_t* n_units, int32_t* sel, int32_t* sel_count,
+                                 float* sel_scores, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
+// Tokens per CTA of the token-level scoring kernels.
+int tok_range(const Derived& d);
 
 // Distant segments per unit the attention kernel may meet for these parameters.
 int64_t max_distant_segments(const Derived& d);

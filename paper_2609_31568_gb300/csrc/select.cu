@@ -203,7 +203,9 @@ constexpr int kTopkThreads = 512;
 
 // One CTA per unit. The k-th largest key T is found with four 8-bit radix
 // passes; the selected blocks are those with key > T plus the lowest-indexed
-// ones with key == T, emitted in ascending block order.
+// ones with key == T, emitted in ascending block order: every thread owns a
+// contiguous span of candidates, counts its picks, and writes them after one
+// block-wide scan of the counts (thread order = index order).
 __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* __restrict__ scores,
                                                        int32_t* __restrict__ sel,
                                                        int32_t* __restrict__ sel_count)
@@ -257,19 +259,29 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
     }
     const uint32_t T = s_prefix;
     const int need_eq = s_need;  // how many keys equal to T to take, lowest b first
-    int taken = 0, eq_seen = 0;
-    for (int64_t base = lo; base < hi; base += blockDim.x) {
-        const int64_t b = base + threadIdx.x;
-        const uint32_t key = (b < hi) ? float_key(sc[b]) : 0u;
-        const int is_eq = (b < hi) && key == T;
-        int eq_total;
-        const int eq_rank = eq_seen + scan_excl(is_eq, sh, &eq_total);
-        const int pick = (b < hi) && (key > T || (is_eq && eq_rank < need_eq));
-        int pick_total;
-        const int pos = taken + scan_excl(pick, sh, &pick_total);
-        if (pick) out[pos] = static_cast<int32_t>(b);
-        taken += pick_total;
-        eq_seen += eq_total;
+    const int64_t span = (n + blockDim.x - 1) / blockDim.x;
+    const int64_t b0 = lo + span * threadIdx.x;
+    const int64_t b1 = (b0 + span < hi) ? b0 + span : hi;
+    int n_gt = 0, n_eq = 0;
+    for (int64_t b = b0; b < b1; ++b) {
+        const uint32_t key = float_key(sc[b]);
+        n_gt += key > T;
+        n_eq += key == T;
+    }
+    int total;
+    const int eq_before = scan_excl(n_eq, sh, &total);
+    int take_eq = need_eq - eq_before;
+    take_eq = take_eq < 0 ? 0 : (take_eq > n_eq ? n_eq : take_eq);
+    int taken;
+    int pos = scan_excl(n_gt + take_eq, sh, &taken);
+    for (int64_t b = b0; b < b1; ++b) {
+        const uint32_t key = float_key(sc[b]);
+        if (key > T) {
+            out[pos++] = static_cast<int32_t>(b);
+        } else if (key == T && take_eq > 0) {
+            out[pos++] = static_cast<int32_t>(b);
+            --take_eq;
+        }
     }
     for (int i = taken + threadIdx.x; i < a.k; i += blockDim.x) out[i] = -1;
     if (threadIdx.x == 0) sel_count[u] = taken;
@@ -317,6 +329,27 @@ cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t
     k_stats<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a, logits, stats);
     k_vote<<<dim3(static_cast<unsigned>((d.nb + 255) / 256), max_units), 256, 0, st>>>(a, logits, stats, scores);
     k_topk<<<max_units, kTopkThreads, 0, st>>>(a, scores, sel_blocks, sel_count);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_end, const float* scores,
+                        int32_t* sel, int32_t* sel_count, cudaStream_t st)
+{
+    SelArgs a{};
+    a.ut = ut;
+    a.sc_begin = sc_begin;
+    a.sc_end = sc_end;
+    a.Hq = d.Hq;
+    a.g = d.g;
+    a.nb = d.nb;
+    a.B = d.B;
+    a.k = d.k;
+    a.n_sink = d.n_sink;
+    a.n_local = d.n_local;
+    a.sigma = d.sigma;
+    const int max_units = sc_end - sc_begin;
+    if (max_units <= 0) return cudaSuccess;
+    k_topk<<<max_units, kTopkThreads, 0, st>>>(a, scores, sel, sel_count);
     return cudaGetLastError();
 }
 

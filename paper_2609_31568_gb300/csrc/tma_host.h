@@ -47,4 +47,28 @@ inline bool make_token_major_map(CUtensorMap* map, const void* base, uint64_t he
     return r == CUDA_SUCCESS;
 }
 
+// A map over a dense bf16 tensor of `rank` dimensions (dims[0] innermost,
+// 128 elements of 2 bytes = 256-byte rows), with 128-byte swizzle and the
+// given box. Returns false on failure.
+inline bool make_dense_bf16_map(CUtensorMap* map, const void* base, uint32_t rank,
+                                const uint64_t* dims, const uint32_t* box)
+{
+    auto enc = tensor_map_encoder();
+    if (!enc || rank < 1 || rank > 5) return false;
+    cuuint64_t d[5], str[4];
+    cuuint32_t b[5], e[5];
+    uint64_t stride = 2;
+    for (uint32_t i = 0; i < rank; ++i) {
+        d[i] = dims[i];
+        b[i] = box[i];
+        e[i] = 1;
+        stride *= dims[i];
+        if (i + 1 < rank) str[i] = stride;
+    }
+    CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), d, str, b,
+                     e, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 }  // namespace scale_host

@@ -107,6 +107,7 @@ def load() -> ctypes.CDLL:
             "scale_build_reps": [pp, P, P, P, P, P, P, P, sz, P],
             "scale_build_reps_noalloc": [pp, P, P, P, P, P, P, P],
             "scale_select": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, sz, P],
+            "scale_select_tokens": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, sz, P],
             "scale_sparse_prefill": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, P, sz, P],
             "scale_get_device_status": [P, P, ctypes.POINTER(i32)],
             "scale_retrieval_calls": [pp, i32, P, i32, ctypes.POINTER(i64), ctypes.POINTER(i64)],
@@ -205,6 +206,14 @@ def scale_select(p, mode, tok_begin, tok_end, reps, fingerprints, unit_start, n_
         _ptr(ws), _nbytes(ws), _stream(stream)))
 
 
+def scale_select_tokens(p, mode, tok_begin, tok_end, k, fingerprints, unit_start, n_units,
+                        sel_tokens, sel_count, sel_scores, ws, stream=None) -> None:
+    _check("scale_select_tokens", load().scale_select_tokens(
+        ctypes.byref(p), mode, tok_begin, tok_end, _ptr(k), _ptr(fingerprints),
+        _ptr(unit_start), _ptr(n_units), _ptr(sel_tokens), _ptr(sel_count), _ptr(sel_scores),
+        _ptr(ws), _nbytes(ws), _stream(stream)))
+
+
 def scale_sparse_prefill(p, mode, tok_begin, tok_end, q, k, v, unit_start, n_units, sel_blocks,
                          sel_count, out, ws, stream=None) -> None:
     _check("scale_sparse_prefill", load().scale_sparse_prefill(
@@ -278,7 +287,8 @@ def allocate(p: ScaleParams, mode: int, device="cuda", want_scores: bool = False
     ws = torch.empty(scale_workspace_size(p, mode), dtype=torch.uint8, device=device)
     scale_workspace_init(ws)
     return Buffers(
-        reps=torch.empty((Hkv, nb, p.head_dim), dtype=f32, device=device),
+        # block size 1 selects from K itself (scale_select_tokens): no representatives
+        reps=None if p.block_size == 1 else torch.empty((Hkv, nb, p.head_dim), dtype=f32, device=device),
         fingerprints=torch.empty((M, Hq * p.head_dim), dtype=f32, device=device),
         unit_start=torch.empty(M + 1, dtype=i32, device=device),
         n_units=torch.empty(1, dtype=i32, device=device),
@@ -290,12 +300,21 @@ def allocate(p: ScaleParams, mode: int, device="cuda", want_scores: bool = False
     )
 
 
+def select(p: ScaleParams, mode: int, tok_begin: int, tok_end: int, k, buf: Buffers, stream=None) -> None:
+    """Steps (b)-(c): block-level selection, or token-level when the block size is 1."""
+    if p.block_size == 1:
+        scale_select_tokens(p, mode, tok_begin, tok_end, k, buf.fingerprints, buf.unit_start,
+                            buf.n_units, buf.sel_blocks, buf.sel_count, buf.sel_scores, buf.ws, stream)
+    else:
+        scale_select(p, mode, tok_begin, tok_end, buf.reps, buf.fingerprints, buf.unit_start,
+                     buf.n_units, buf.sel_blocks, buf.sel_count, buf.sel_scores, buf.ws, stream)
+
+
 def run_path(p: ScaleParams, mode: int, q, k, v, buf: Buffers, tok_begin: int = 0,
              tok_end: int | None = None, stream=None) -> None:
     """Steps (a)-(d) on one layer: build reps and clusters, select, attend."""
     tok_end = p.n_tokens if tok_end is None else tok_end
     scale_build_reps(p, q, k, buf.reps, buf.fingerprints, buf.unit_start, buf.n_units, buf.ws, stream)
-    scale_select(p, mode, tok_begin, tok_end, buf.reps, buf.fingerprints, buf.unit_start,
-                 buf.n_units, buf.sel_blocks, buf.sel_count, buf.sel_scores, buf.ws, stream)
+    select(p, mode, tok_begin, tok_end, k, buf, stream)
     scale_sparse_prefill(p, mode, tok_begin, tok_end, q, k, v, buf.unit_start, buf.n_units,
                          buf.sel_blocks, buf.sel_count, buf.out, buf.ws, stream)

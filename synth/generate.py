@@ -111,6 +111,12 @@ WORKLOADS: dict[str, Workload] = {
 }
 
 
+# Token-level selection (block size 1, the paper's own rule) with the paper's
+# k = 8192 tokens, on the 128K and 1M layers.
+WORKLOADS["llama8b-128k-tok"] = WORKLOADS["llama8b-128k"].replace(name="llama8b-128k-tok", block_size=1,
+                                                                 top_k=8192)
+WORKLOADS["llama8b-1m-tok"] = WORKLOADS["llama8b-1m"].replace(name="llama8b-1m-tok", block_size=1, top_k=8192)
+
 # Planted-topic variant for the clustering-threshold sweep: the paper's sub-chunk
 # L = 512 and outer chunk 8192, k = 64 blocks of 128 = 8192 tokens, 128K context.
 WORKLOADS["llama8b-128k-topics"] = Workload(

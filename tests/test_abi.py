@@ -134,3 +134,27 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(S, "_lib", None)
     with pytest.raises(S.ScaleLibraryMissing):
         S.load()
+
+
+def test_block_and_token_selection_entry_points_check_block_size(lib):
+    """scale_select serves block sizes > 1, scale_select_tokens block size 1;
+    each refuses the other before looking at any pointer."""
+    p1 = S.params_for(workload("llama8b-32k", block_size=1, top_k=1024))
+    assert lib.scale_select(ctypes.byref(p1), 0, 0, p1.n_tokens, None, None, None, None, None, None,
+                            None, None, 0, None) == S.SCALE_ERR_UNSUPPORTED
+    pb = _p()
+    assert lib.scale_select_tokens(ctypes.byref(pb), 0, 0, pb.n_tokens, None, None, None, None, None,
+                                   None, None, None, 0, None) == S.SCALE_ERR_INVALID_ARG
+    p16 = S.params_for(workload("llama8b-32k", block_size=1, num_kv_heads=2))  # 16 query heads per KV head
+    assert lib.scale_select_tokens(ctypes.byref(p16), 0, 0, p16.n_tokens, None, None, None, None, None,
+                                   None, None, None, 0, None) == S.SCALE_ERR_UNSUPPORTED
+
+
+def test_token_workspace_has_no_logits_plane():
+    """Block size 1 keeps no [units][heads][tokens] logits (that would be 32 GB
+    at 1M tokens per sub-chunk); the scores plane [units][tokens] remains."""
+    p = S.params_for(workload("llama8b-1m-tok"))
+    n = S.scale_workspace_size(p, S.SCALE_MODE_PER_SUBCHUNK)
+    M, N = 256, 1 << 20
+    assert M * N * 4 <= n < M * N * 4 * 1.3
+

@@ -229,6 +229,92 @@ def test_end_to_end_parity_sampled(name, n_random, mode):
     assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
 
 
+# --------------------------------------------------------------------------- token level (B = 1)
+
+TOKEN_CASES = [("gqa4-4k", dict(block_size=1, top_k=64)),
+               ("gqa4-4k", dict(block_size=1, n_tokens=3000, n_sink=40, n_local=100, top_k=50)),
+               ("llama8b-32k", dict(block_size=1, top_k=1024))]
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+@pytest.mark.parametrize("name,over", TOKEN_CASES + [("llama8b-128k-tok", {})])
+def test_token_select_parity(name, over, mode):
+    """scale_select_tokens (tensor-core scores from K, per-head softmax, soft
+    vote, top-k of tokens) against the oracle's Eq. 9 at block size 1."""
+    w, q, k, v, dev = inputs(name, **over)
+    p, buf = gpu_path(w, mode, dev)
+    ref = oracle.run_path(w, q, k, v, per_subchunk=(mode == PER_SUB))
+    n = unit_count(buf, mode, w)
+    sel = buf.sel_blocks.cpu().numpy()[:n, : w.top_k]
+    cnt = buf.sel_count.cpu().numpy()[:n]
+    same, near = compare_selection(sel, cnt, ref)
+    ref_sc = oracle.select(num_q_heads=w.num_q_heads, n_tokens=w.n_tokens, sub_chunk=w.sub_chunk,
+                           block_size=1, top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                           select_scale=1.0, per_subchunk=(mode == PER_SUB), reps=ref["reps"],
+                           v=ref["fingerprints"], unit_start=ref["unit_start"], want_scores=True)["scores"]
+    got_sc = buf.sel_scores.cpu().numpy()[:n].astype(np.float64)
+    cand = ~np.isnan(ref_sc)
+    assert np.array_equal(cand, ~np.isnan(got_sc))
+    np.testing.assert_allclose(got_sc[cand], ref_sc[cand], rtol=2e-5, atol=1e-10)
+    print(f"{name} {over} mode={mode}: {n} units, {near} near-tie units differ")
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+@pytest.mark.parametrize("name,over,stride", [(nm, ov, 1 if nm == "gqa4-4k" else 5) for nm, ov in TOKEN_CASES])
+def test_token_attention_parity_on_oracle_selection(name, over, stride, mode):
+    """scale_sparse_prefill at block size 1 (distant keys gathered row by row)
+    on the oracle's token selection vs the oracle's Eq. 10."""
+    w, q, k, v, dev = inputs(name, **over)
+    rows = np.arange(0, w.n_tokens, stride)
+    ref = oracle_path(w, q, k, v, mode, rows=rows)
+    us = ref["unit_start"] if mode == PER_CLUSTER else np.arange(w.n_subchunks + 1, dtype=np.int32)
+    out = _prefill_on(w, mode, dev, us, len(us) - 1, ref["sel"], ref["sel_count"])
+    got = to_f64_bf16(out[torch.from_numpy(rows).cuda()])
+    mx, mean = attn_errors(got, ref["attn"])
+    print(f"{name} {over} mode={mode}: max {mx:.3e} mean {mean:.3e}")
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+def test_token_attention_ignores_invalid_entries():
+    """Selected tokens outside [n_sink, W_u), repeated or out of order are
+    ignored, as scale_sparse_prefill documents: the result equals the one on
+    the cleaned selection."""
+    w, q, k, v, dev = inputs("gqa4-4k", block_size=1, top_k=64)
+    ref = oracle_path(w, q, k, v, PER_CLUSTER)
+    us = ref["unit_start"]
+    clean = _prefill_on(w, PER_CLUSTER, dev, us, len(us) - 1, ref["sel"], ref["sel_count"])
+    dirty = ref["sel"].copy()
+    cnt = ref["sel_count"].copy()
+    for u in range(len(cnt)):
+        c = int(cnt[u])
+        if c >= 4:
+            dirty[u, 1] = dirty[u, 0]          # repeat (not above its predecessor)
+            dirty[u, c - 1] = w.n_tokens + 5   # beyond the window
+    bad = _prefill_on(w, PER_CLUSTER, dev, us, len(us) - 1, dirty, cnt)
+    cleaned = [[t for i, t in enumerate(dirty[u, : cnt[u]])
+                if w.n_sink <= t < max(0, us[u] * w.sub_chunk - w.n_local) and (i == 0 or t > dirty[u, i - 1])]
+               for u in range(len(cnt))]
+    sel2 = np.full_like(dirty, -1)
+    cnt2 = np.array([len(x) for x in cleaned], np.int32)
+    for u, x in enumerate(cleaned):
+        sel2[u, : len(x)] = x
+    ref2 = _prefill_on(w, PER_CLUSTER, dev, us, len(us) - 1, sel2, cnt2)
+    assert torch.equal(bad, ref2)
+    assert not torch.equal(bad, clean)
+
+
+def test_1m_tokens_full_size():
+    """Token-level selection at 1M tokens with k = 8192 (SCR): every unit's
+    selection and sampled attention rows against the oracle."""
+    from synth import generate_layer, workload
+
+    w = workload("llama8b-1m-tok")
+    q, k, v = generate_layer(w)
+    n, mx, mean, near = _full_size_check(w, q, k, v, PER_CLUSTER, n_random=24)
+    print(f"1M tokens: {n} rows, max {mx:.3e} mean {mean:.3e}, {near} near-tie units")
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
 # --------------------------------------------------------------------------- threshold sweep
 
 
