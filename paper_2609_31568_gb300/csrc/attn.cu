@@ -70,9 +70,8 @@ struct AttnArgs {
     float scale_log2;
     const int32_t* sel;
     const int32_t* sel_count;
-    const int32_t* tok_list;   // block size 1: [M][list_stride] distant tokens of each unit
-    const int32_t* tok_count;  // block size 1: [M] entries of each list
-    int list_stride;
+    const int32_t* tok_count;  // block size 1: [M] distant keys of each unit (packed)
+    int slots;                 // block size 1: packed rows per (unit, KV head), a multiple of 128
     __nv_bfloat16* out;
     int32_t* status;
     uint64_t timeout_ns;
@@ -93,15 +92,15 @@ __device__ __forceinline__ void fail(volatile int* abort_flag, int32_t* status)
     record_status(status, SCALE_ERR_TIMEOUT);
 }
 
-// TOK: block size 1. The distant keys of a unit are the token list built by
-// k_tok_lists; tiles of it are gathered row by row (TMA gather4, four rows per
-// instruction, all 32 lanes of the producer warp issuing) through 2-D maps
-// over K and V viewed as [N * H_kv][128].
+// TOK: block size 1. The distant keys and values of each (unit, KV head)
+// were packed by k_tok_pack into contiguous rows [M * H_kv][slots][128]
+// (zero rows after the last one), so their tiles are plain TMA boxes of the
+// maps tpk / tpv, like the window's.
 template <bool TOK>
 __global__ void __launch_bounds__(kThreads, 1)
 k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CUtensorMap tk,
-              const __grid_constant__ CUtensorMap tv, const __grid_constant__ CUtensorMap tgk,
-              const __grid_constant__ CUtensorMap tgv, const AttnArgs a)
+              const __grid_constant__ CUtensorMap tv, const __grid_constant__ CUtensorMap tpk,
+              const __grid_constant__ CUtensorMap tpv, const AttnArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ Barriers bars;
@@ -165,7 +164,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     if (TOK && warp == 8) {
         if (lane == 0) {
             int n = a.tok_count[u];
-            n = n < 0 ? 0 : (n > a.list_stride ? a.list_stride : n);
+            n = n < 0 ? 0 : (n > a.slots ? a.slots : n);
             s_nseg = n;  // distant tokens (not segments) in this mode
         }
     } else if (warp == 8) {
@@ -228,102 +227,76 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
 
     if (warp == 8) {
         // ------------------------------------------------------------ producer
-        // The whole warp walks the tiles; lane 0 waits and arms the barriers,
-        // and issues the box loads; gathered tiles are issued by all lanes.
         if (lane == 0) {
             tma_prefetch_desc(&tq);
             tma_prefetch_desc(&tk);
             tma_prefetch_desc(&tv);
             if (TOK) {
-                tma_prefetch_desc(&tgk);
-                tma_prefetch_desc(&tgv);
+                tma_prefetch_desc(&tpk);
+                tma_prefetch_desc(&tpv);
             }
             mbar_arrive_expect_tx(&bars.q_full, 2 * kTileBytes);
             for (int qt = 0; qt < 2; ++qt)
                 for (int hf = 0; hf < 2; ++hf)
                     tma_load_3d(smem + kOffQ + qt * kTileBytes + hf * kHalf, &tq, &bars.q_full,
                                 hf * 64, h0 + qt, static_cast<int32_t>(q0));
-        }
-        int issued_k0 = 0, issued_k1 = 0, issued_v0 = 0, issued_v1 = 0;
-        const int32_t* list = TOK ? a.tok_list + static_cast<int64_t>(u) * a.list_stride : nullptr;
-        for (int t = 0; t < T; ++t) {
-            const int st = t & 1;
-            const uint32_t ph = ((t >> 1) - 1) & 1;
-            const bool gather = TOK && t < n_dt;
-            int32_t ta = 0, tb = 0;
-            int32_t rows[4] = {0, 0, 0, 0};
-            if (gather) {
-#pragma unroll
-                for (int m = 0; m < 4; ++m) {
-                    const int slot = 128 * t + 4 * lane + m;
-                    const int tok = slot < s_nseg ? list[slot] : 0;  // padding: a valid row, masked
-                    rows[m] = tok * a.Hkv + kvh;
+            const int32_t prow = u * a.Hkv + kvh;  // packed (unit, KV head) plane
+            int issued_k0 = 0, issued_k1 = 0, issued_v0 = 0, issued_v1 = 0;
+            for (int t = 0; t < T && !abort_flag; ++t) {
+                const int st = t & 1;
+                const uint32_t ph = ((t >> 1) - 1) & 1;
+                const bool packed = TOK && t < n_dt;
+                int32_t ta, tb;
+                if (packed) {
+                    ta = 128 * t;
+                    tb = 0;
+                } else if (t < n_dt) {
+                    ta = seg[2 * t].x;
+                    tb = seg[2 * t + 1].x;
+                } else {
+                    ta = static_cast<int32_t>(W + 128ll * (t - n_dt));
+                    tb = ta + 64;
                 }
-            } else if (t < n_dt) {
-                ta = seg[2 * t].x;
-                tb = seg[2 * t + 1].x;
-            } else {
-                ta = static_cast<int32_t>(W + 128ll * (t - n_dt));
-                tb = ta + 64;
-            }
-            // K tile
-            int ok = 1;
-            if (lane == 0) {
-                ok = !abort_flag;
-                if (ok && t >= 2 && !mbar_wait_bounded(&bars.k_empty[st], ph, a.timeout_ns, &abort_flag)) {
+                if (t >= 2 && !mbar_wait_bounded(&bars.k_empty[st], ph, a.timeout_ns, &abort_flag)) {
                     fail(&abort_flag, a.status);
-                    ok = 0;
+                    break;
                 }
-                if (ok) {
-                    mbar_arrive_expect_tx(&bars.k_full[st], kTileBytes);
-                    if (st) ++issued_k1; else ++issued_k0;
-                }
-            }
-            if (!__shfl_sync(0xFFFFFFFFu, ok, 0)) break;
-            uint8_t* kd = smem + kOffK + st * kTileBytes;
-            if (gather) {
-                for (int hf = 0; hf < 2; ++hf)
-                    tma_gather4(kd + hf * kHalf + lane * 512, &tgk, &bars.k_full[st], hf * 64, rows[0],
-                                rows[1], rows[2], rows[3]);
-            } else if (lane == 0) {
+                mbar_arrive_expect_tx(&bars.k_full[st], kTileBytes);
+                if (st) ++issued_k1; else ++issued_k0;
+                uint8_t* kd = smem + kOffK + st * kTileBytes;
                 for (int hf = 0; hf < 2; ++hf) {
-                    tma_load_3d(kd + hf * kHalf, &tk, &bars.k_full[st], hf * 64, kvh, ta);
-                    tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.k_full[st], hf * 64, kvh, tb);
+                    if (packed) {
+                        tma_load_3d(kd + hf * kHalf, &tpk, &bars.k_full[st], hf * 64, ta, prow);
+                    } else {
+                        tma_load_3d(kd + hf * kHalf, &tk, &bars.k_full[st], hf * 64, kvh, ta);
+                        tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.k_full[st], hf * 64, kvh, tb);
+                    }
                 }
-            }
-            // V tile
-            if (lane == 0) {
-                ok = !abort_flag;
-                if (ok && t >= 2 && !mbar_wait_bounded(&bars.v_empty[st], ph, a.timeout_ns, &abort_flag)) {
+                if (t >= 2 && !mbar_wait_bounded(&bars.v_empty[st], ph, a.timeout_ns, &abort_flag)) {
                     fail(&abort_flag, a.status);
-                    ok = 0;
+                    break;
                 }
-                if (ok) {
-                    mbar_arrive_expect_tx(&bars.v_full[st], kTileBytes);
-                    if (st) ++issued_v1; else ++issued_v0;
-                }
-            }
-            if (!__shfl_sync(0xFFFFFFFFu, ok, 0)) break;
-            uint8_t* vd = smem + kOffV + st * kTileBytes;
-            if (gather) {
-                for (int hf = 0; hf < 2; ++hf)
-                    tma_gather4(vd + hf * kHalf + lane * 512, &tgv, &bars.v_full[st], hf * 64, rows[0],
-                                rows[1], rows[2], rows[3]);
-            } else if (lane == 0) {
+                mbar_arrive_expect_tx(&bars.v_full[st], kTileBytes);
+                if (st) ++issued_v1; else ++issued_v0;
+                uint8_t* vd = smem + kOffV + st * kTileBytes;
                 for (int hf = 0; hf < 2; ++hf) {
-                    tma_load_3d(vd + hf * kHalf, &tv, &bars.v_full[st], hf * 64, kvh, ta);
-                    tma_load_3d(vd + hf * kHalf + kSegBytes, &tv, &bars.v_full[st], hf * 64, kvh, tb);
+                    if (packed) {
+                        tma_load_3d(vd + hf * kHalf, &tpv, &bars.v_full[st], hf * 64, ta, prow);
+                    } else {
+                        tma_load_3d(vd + hf * kHalf, &tv, &bars.v_full[st], hf * 64, kvh, ta);
+                        tma_load_3d(vd + hf * kHalf + kSegBytes, &tv, &bars.v_full[st], hf * 64, kvh, tb);
+                    }
                 }
             }
-        }
-        if (lane == 0 && abort_flag) {
-            // Drain: wait (bounded, ignoring the abort flag) for the last
-            // phase of every buffer that received copies.
-            mbar_wait_bounded(&bars.q_full, 0, a.timeout_ns, nullptr);
-            if (issued_k0) mbar_wait_bounded(&bars.k_full[0], (issued_k0 - 1) & 1, a.timeout_ns, nullptr);
-            if (issued_k1) mbar_wait_bounded(&bars.k_full[1], (issued_k1 - 1) & 1, a.timeout_ns, nullptr);
-            if (issued_v0) mbar_wait_bounded(&bars.v_full[0], (issued_v0 - 1) & 1, a.timeout_ns, nullptr);
-            if (issued_v1) mbar_wait_bounded(&bars.v_full[1], (issued_v1 - 1) & 1, a.timeout_ns, nullptr);
+            if (abort_flag) {
+                // Drain: wait (bounded, ignoring the abort flag) for the last
+                // phase of every buffer that received copies.
+                mbar_wait_bounded(&bars.q_full, 0, a.timeout_ns, nullptr);
+                if (issued_k0) mbar_wait_bounded(&bars.k_full[0], (issued_k0 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_k1) mbar_wait_bounded(&bars.k_full[1], (issued_k1 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_v0) mbar_wait_bounded(&bars.v_full[0], (issued_v0 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_v1) mbar_wait_bounded(&bars.v_full[1], (issued_v1 - 1) & 1, a.timeout_ns, nullptr);
+            }
         }
     } else if (warp == 9) {
         // ------------------------------------------------------------ MMA issuer
@@ -402,7 +375,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
             tmem_ld_wait();
             float* s = reinterpret_cast<float*>(sr);
             if (TOK && t < n_dt) {
-                const int lim = s_nseg - 128 * t;  // gathered slots past the list are padding
+                const int lim = s_nseg - 128 * t;  // packed rows past the list are zero padding
                 if (lim < 128) {
 #pragma unroll
                     for (int c = 0; c < 128; ++c)
@@ -521,43 +494,68 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     }
 }
 
-// Block size 1: the distant key list of every unit, one warp per unit: the
-// sinks [0, min(n_sink, W_u)), then every selected token in [n_sink, W_u)
-// that is larger than the entry before it (so each key appears once, in
-// ascending order). Writes the list and its length.
-__global__ void __launch_bounds__(32) k_tok_lists(Units ut, int sc_begin, int sc_end, int n_sink,
-                                                  int n_local, int k, const int32_t* __restrict__ sel,
+// Block size 1: pack the distant keys and values of unit u (blockIdx.x) and
+// KV head blockIdx.y into contiguous rows: the sinks [0, min(n_sink, W_u)),
+// then every selected token in [n_sink, W_u) that is larger than the entry
+// before it (each key once, ascending); zero rows up to the next multiple of
+// 128. Writes the number of keys of each unit.
+__global__ void __launch_bounds__(256) k_tok_pack(Units ut, int sc_begin, int sc_end, int n_sink, int n_local,
+                                                  int k, int Hkv, const int32_t* __restrict__ sel,
                                                   const int32_t* __restrict__ sel_count,
-                                                  int32_t* __restrict__ list, int32_t* __restrict__ count,
-                                                  int stride)
+                                                  const uint4* __restrict__ kin, const uint4* __restrict__ vin,
+                                                  uint4* __restrict__ kout, uint4* __restrict__ vout,
+                                                  int32_t* __restrict__ count, int slots)
 {
+    extern __shared__ int32_t s_list[];  // [slots]
+    __shared__ int s_n;
     const int u = unit_lower_bound(ut, sc_begin) + static_cast<int>(blockIdx.x);
     if (u >= unit_lower_bound(ut, sc_end)) return;
-    int anchor;
-    int64_t s_u, e_u;
-    unit_range(ut, u, &anchor, &s_u, &e_u);
-    const int64_t W = (s_u - n_local > 0) ? s_u - n_local : 0;
-    const int lane = threadIdx.x;
-    int32_t* out = list + static_cast<int64_t>(u) * stride;
-    const int n_s = static_cast<int>(n_sink < W ? n_sink : W);
-    for (int i = lane; i < n_s; i += 32) out[i] = i;
-    int base = n_s;
-    int cnt = sel_count[u];
-    cnt = cnt < 0 ? 0 : (cnt > k ? k : cnt);
-    const int32_t* sl = sel + static_cast<int64_t>(u) * k;
-    for (int c0 = 0; c0 < cnt; c0 += 32) {
-        const int i = c0 + lane;
-        bool valid = false;
-        int32_t tok = 0;
-        if (i < cnt) {
-            tok = sl[i];
-            valid = tok >= n_sink && tok < W && (i == 0 || tok > sl[i - 1]);
+    const int kvh = blockIdx.y;
+    const int tid = threadIdx.x, lane = tid & 31;
+    if (tid < 32) {
+        int anchor;
+        int64_t s_u, e_u;
+        unit_range(ut, u, &anchor, &s_u, &e_u);
+        const int64_t W = (s_u - n_local > 0) ? s_u - n_local : 0;
+        const int n_s = static_cast<int>(n_sink < W ? n_sink : W);
+        for (int i = lane; i < n_s; i += 32) s_list[i] = i;
+        int base = n_s;
+        int cnt = sel_count[u];
+        cnt = cnt < 0 ? 0 : (cnt > k ? k : cnt);
+        const int32_t* sl = sel + static_cast<int64_t>(u) * k;
+        for (int c0 = 0; c0 < cnt; c0 += 32) {
+            const int i = c0 + lane;
+            bool valid = false;
+            int32_t tok = 0;
+            if (i < cnt) {
+                tok = sl[i];
+                valid = tok >= n_sink && tok < W && (i == 0 || tok > sl[i - 1]);
+            }
+            const uint32_t b = __ballot_sync(0xFFFFFFFFu, valid);
+            if (valid) s_list[base + __popc(b & ((1u << lane) - 1u))] = tok;
+            base += __popc(b);
         }
-        const uint32_t b = __ballot_sync(0xFFFFFFFFu, valid);
-        if (valid) out[base + __popc(b & ((1u << lane) - 1u))] = tok;
-        base += __popc(b);
+        if (lane == 0) {
+            s_n = base;
+            if (kvh == 0) count[u] = base;
+        }
     }
-    if (lane == 0) count[u] = base;
+    __syncthreads();
+    const int n = s_n;
+    const int n_pad = (n + 127) / 128 * 128;
+    const int64_t plane = (static_cast<int64_t>(u) * Hkv + kvh) * slots * 16;  // 16-byte chunks
+    const uint4 zero = make_uint4(0, 0, 0, 0);
+    for (int i = tid; i < n_pad * 16; i += blockDim.x) {
+        const int slot = i >> 4, c = i & 15;
+        uint4 kx = zero, vx = zero;
+        if (slot < n) {
+            const int64_t src = (static_cast<int64_t>(s_list[slot]) * Hkv + kvh) * 16 + c;
+            kx = kin[src];
+            vx = vin[src];
+        }
+        kout[plane + i] = kx;
+        vout[plane + i] = vx;
+    }
 }
 
 // Bounded-wait self-check: wait on a barrier nothing arrives at.
@@ -577,6 +575,11 @@ __global__ void k_wait_selftest(int32_t* status, uint64_t timeout_ns)
 
 }  // namespace
 
+int tok_slots(const Derived& d)
+{
+    return (d.n_sink + d.k + 127) / 128 * 128;
+}
+
 int64_t max_distant_segments(const Derived& d)
 {
     // ceil(n_sink / 64) sink segments, at most ceil(B / 64) per selected block,
@@ -590,22 +593,24 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
                                   const int32_t* sel_blocks, const int32_t* sel_count, void* out,
                                   uint8_t* ws, uint64_t timeout_ns, cudaStream_t st)
 {
-    CUtensorMap tq, tk, tv, tgk, tgv;
+    CUtensorMap tq, tk, tv, tpk, tpv;
     if (!scale_host::make_token_major_map(&tq, q, kHeadDim, d.Hq, d.N, 64, 128) ||
         !scale_host::make_token_major_map(&tk, k, kHeadDim, d.Hkv, d.N, 64, 64) ||
         !scale_host::make_token_major_map(&tv, v, kHeadDim, d.Hkv, d.N, 64, 64))
         return cudaErrorInvalidValue;
     const bool tok = d.B == 1;
+    const WsLayout lay = ws_layout(d);
+    const int slots = tok_slots(d);
     if (tok) {
-        // K and V as [N * H_kv] rows of 128, one-row boxes of 64 columns (gather4)
-        const uint64_t gdims[2] = {kHeadDim, static_cast<uint64_t>(d.N) * d.Hkv};
-        const uint32_t gbox[2] = {64, 1};
-        if (!scale_host::make_dense_bf16_map(&tgk, k, 2, gdims, gbox) ||
-            !scale_host::make_dense_bf16_map(&tgv, v, 2, gdims, gbox))
+        // packed distant rows [M * H_kv][slots][128], boxes of 64 x 128 rows
+        const uint64_t pdims[3] = {kHeadDim, static_cast<uint64_t>(slots), static_cast<uint64_t>(d.M) * d.Hkv};
+        const uint32_t pbox[3] = {64, 128, 1};
+        if (!scale_host::make_dense_bf16_map(&tpk, ws + lay.tok_pack_k, 3, pdims, pbox) ||
+            !scale_host::make_dense_bf16_map(&tpv, ws + lay.tok_pack_v, 3, pdims, pbox))
             return cudaErrorInvalidValue;
     } else {
-        tgk = tk;
-        tgv = tv;
+        tpk = tk;
+        tpv = tv;
     }
 
     AttnArgs a;
@@ -629,25 +634,30 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
     a.scale_log2 = d.attn_scale * 1.4426950408889634f;
     a.sel = sel_blocks;
     a.sel_count = sel_count;
-    const WsLayout lay = ws_layout(d);
-    a.tok_list = tok ? reinterpret_cast<const int32_t*>(ws + lay.tok_list) : nullptr;
     a.tok_count = tok ? reinterpret_cast<const int32_t*>(ws + lay.tok_count) : nullptr;
-    a.list_stride = d.n_sink + d.k;
+    a.slots = slots;
     a.out = static_cast<__nv_bfloat16*>(out);
     a.status = reinterpret_cast<int32_t*>(ws + kStatusOffset);
     a.timeout_ns = timeout_ns;
 
-    if (tok)
-        k_tok_lists<<<a.n_sc, 32, 0, st>>>(a.ut, a.sc_begin, a.sc_end, d.n_sink, d.n_local, d.k, sel_blocks,
-                                           sel_count, const_cast<int32_t*>(a.tok_list),
-                                           const_cast<int32_t*>(a.tok_count), a.list_stride);
+    if (tok) {
+        const size_t list_bytes = static_cast<size_t>(slots) * sizeof(int32_t);
+        cudaError_t e = cudaFuncSetAttribute(k_tok_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(list_bytes));
+        if (e != cudaSuccess) return e;
+        k_tok_pack<<<dim3(a.n_sc, d.Hkv), 256, list_bytes, st>>>(
+            a.ut, a.sc_begin, a.sc_end, d.n_sink, d.n_local, d.k, d.Hkv, sel_blocks, sel_count,
+            static_cast<const uint4*>(k), static_cast<const uint4*>(v),
+            reinterpret_cast<uint4*>(ws + lay.tok_pack_k), reinterpret_cast<uint4*>(ws + lay.tok_pack_v),
+            const_cast<int32_t*>(a.tok_count), slots);
+    }
     auto kern = tok ? k_sparse_attn<true> : k_sparse_attn<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(kSmemBytes));
     if (e != cudaSuccess) return e;
     const int64_t grid = static_cast<int64_t>(a.n_sc) * a.qb_per_sc * d.Hkv * a.pairs;
     if (grid <= 0 || grid > 0x7FFFFFFFll) return cudaErrorInvalidConfiguration;
-    kern<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tq, tk, tv, tgk, tgv, a);
+    kern<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, st>>>(tq, tk, tv, tpk, tpv, a);
     return cudaGetLastError();
 }
 

@@ -46,8 +46,9 @@ struct WsLayout {
     size_t logits;      // fp32 [M][H_q][nb]     (block size > 1 only)
     size_t tok_split;   // bf16 [3][H_kv][M][g][128]  fingerprint parts (block size 1 only)
     size_t tok_part;    // float2 [M][H_q][ranges]    per-range softmax partials (block size 1 only)
-    size_t tok_list;    // int32 [M][n_sink + k]      distant token list per unit (block size 1 only)
-    size_t tok_count;   // int32 [M]                  its length
+    size_t tok_pack_k;  // bf16 [M][H_kv][slots][128] distant keys of each unit, packed (block size 1 only)
+    size_t tok_pack_v;  // bf16 [M][H_kv][slots][128] distant values, packed
+    size_t tok_count;   // int32 [M]                  distant keys of each unit
     size_t stats;       // fp32 [M][H_q][2]  (row max, 1 / row sum)
     size_t scores;      // fp32 [M][nb]
     size_t total;
@@ -138,6 +139,10 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
                                  float* sel_scores, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 // Tokens per CTA of the token-level scoring kernels.
 int tok_range(const Derived& d);
+
+// Packed distant rows per (unit, KV head) at block size 1: n_sink + k rounded
+// up to a multiple of 128.
+int tok_slots(const Derived& d);
 
 // Distant segments per unit the attention kernel may meet for these parameters.
 int64_t max_distant_segments(const Derived& d);

@@ -152,9 +152,13 @@ def test_block_and_token_selection_entry_points_check_block_size(lib):
 
 def test_token_workspace_has_no_logits_plane():
     """Block size 1 keeps no [units][heads][tokens] logits (that would be 32 GB
-    at 1M tokens per sub-chunk); the scores plane [units][tokens] remains."""
-    p = S.params_for(workload("llama8b-1m-tok"))
+    at 1M tokens per sub-chunk): the workspace is the [units][tokens] scores
+    plus the packed distant keys and values of every unit, plus small parts."""
+    w = workload("llama8b-1m-tok")
+    p = S.params_for(w)
     n = S.scale_workspace_size(p, S.SCALE_MODE_PER_SUBCHUNK)
-    M, N = 256, 1 << 20
-    assert M * N * 4 <= n < M * N * 4 * 1.3
-
+    M, N = w.n_subchunks, w.n_tokens
+    slots = -(-(w.n_sink + w.top_k) // 128) * 128
+    big = M * N * 4 + 2 * M * w.num_kv_heads * slots * 128 * 2
+    assert big <= n < big * 1.1
+    assert n < M * w.num_q_heads * N * 4  # the logits plane alone would be larger
