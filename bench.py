@@ -75,7 +75,7 @@ def launches(w, selects: int = 1) -> dict:
     tok = w.block_size == 1
     build = (3 if tok else 4) + (1 if w.max_cluster_subchunks > 1 else 0)
     select = 5 if tok else 4
-    attend = 2 if tok else 1
+    attend = 3 if tok else 1
     return {"build_reps": build, "select": select * selects, "attend": attend * selects,
             "total": build + (select + attend) * selects}
 

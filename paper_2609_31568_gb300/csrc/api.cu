@@ -71,6 +71,7 @@ WsLayout ws_layout(const Derived& d)
     const int64_t ranges = tok ? (d.N + tok_range(d) - 1) / tok_range(d) : 0;
     w.tok_part = take(static_cast<size_t>(d.M) * d.Hq * ranges * 2 * sizeof(float));
     const size_t pack = tok ? static_cast<size_t>(d.M) * d.Hkv * tok_slots(d) * kHeadDim * 2 : 0;
+    w.tok_list = take(tok ? static_cast<size_t>(d.M) * tok_slots(d) * sizeof(int32_t) : 0);
     w.tok_pack_k = take(pack);
     w.tok_pack_v = take(pack);
     w.tok_count = take(tok ? static_cast<size_t>(d.M) * sizeof(int32_t) : 0);
@@ -256,7 +257,6 @@ int scale_sparse_prefill(const scale_params_t* p, int32_t mode, int64_t tok_begi
     if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
     if (d.g % 2) return SCALE_ERR_UNSUPPORTED;
     if (d.B > 1 && max_distant_segments(d) > kMaxSegments) return SCALE_ERR_UNSUPPORTED;
-    if (d.B == 1 && static_cast<int64_t>(tok_slots(d)) * 4 > 200 * 1024) return SCALE_ERR_UNSUPPORTED;
     if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(v, 16) || !device_ptr(out, 16) ||
         !device_ptr(sel_count, 4) || (d.k > 0 && !device_ptr(sel_blocks, 4)))
         return SCALE_ERR_INVALID_ARG;

@@ -494,62 +494,71 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     }
 }
 
-// Block size 1: pack the distant keys and values of unit u (blockIdx.x) and
-// KV head blockIdx.y into contiguous rows: the sinks [0, min(n_sink, W_u)),
-// then every selected token in [n_sink, W_u) that is larger than the entry
-// before it (each key once, ascending); zero rows up to the next multiple of
-// 128. Writes the number of keys of each unit.
-__global__ void __launch_bounds__(256) k_tok_pack(Units ut, int sc_begin, int sc_end, int n_sink, int n_local,
-                                                  int k, int Hkv, const int32_t* __restrict__ sel,
+// Block size 1, step 1 of 2: the distant list of every unit, one warp per
+// unit: the sinks [0, min(n_sink, W_u)), then every selected token in
+// [n_sink, W_u) larger than the entry before it (each key once, ascending).
+__global__ void __launch_bounds__(32) k_tok_lists(Units ut, int sc_begin, int sc_end, int n_sink, int n_local,
+                                                  int k, const int32_t* __restrict__ sel,
                                                   const int32_t* __restrict__ sel_count,
-                                                  const uint4* __restrict__ kin, const uint4* __restrict__ vin,
-                                                  uint4* __restrict__ kout, uint4* __restrict__ vout,
-                                                  int32_t* __restrict__ count, int slots)
+                                                  int32_t* __restrict__ list, int32_t* __restrict__ count, int slots)
 {
-    extern __shared__ int32_t s_list[];  // [slots]
-    __shared__ int s_n;
+    const int u = unit_lower_bound(ut, sc_begin) + static_cast<int>(blockIdx.x);
+    if (u >= unit_lower_bound(ut, sc_end)) return;
+    const int lane = threadIdx.x;
+    int anchor;
+    int64_t s_u, e_u;
+    unit_range(ut, u, &anchor, &s_u, &e_u);
+    const int64_t W = (s_u - n_local > 0) ? s_u - n_local : 0;
+    int32_t* out = list + static_cast<int64_t>(u) * slots;
+    const int n_s = static_cast<int>(n_sink < W ? n_sink : W);
+    for (int i = lane; i < n_s; i += 32) out[i] = i;
+    int base = n_s;
+    int cnt = sel_count[u];
+    cnt = cnt < 0 ? 0 : (cnt > k ? k : cnt);
+    const int32_t* sl = sel + static_cast<int64_t>(u) * k;
+    for (int c0 = 0; c0 < cnt; c0 += 32) {
+        const int i = c0 + lane;
+        bool valid = false;
+        int32_t tok = 0;
+        if (i < cnt) {
+            tok = sl[i];
+            valid = tok >= n_sink && tok < W && (i == 0 || tok > sl[i - 1]);
+        }
+        const uint32_t b = __ballot_sync(0xFFFFFFFFu, valid);
+        if (valid) out[base + __popc(b & ((1u << lane) - 1u))] = tok;
+        base += __popc(b);
+    }
+    if (lane == 0) count[u] = base;
+}
+
+// Block size 1, step 2 of 2: copy the listed K and V rows of unit u
+// (blockIdx.x) and KV head blockIdx.y, slots [256 z, 256 z + 256) with
+// z = blockIdx.z, into contiguous rows [M * H_kv][slots][128]; slots past the
+// list up to the next multiple of 128 are written as zeros.
+constexpr int kPackSlots = 256;
+__global__ void __launch_bounds__(256) k_tok_pack(Units ut, int sc_begin, int sc_end, int Hkv,
+                                                  const int32_t* __restrict__ list,
+                                                  const int32_t* __restrict__ count,
+                                                  const uint4* __restrict__ kin, const uint4* __restrict__ vin,
+                                                  uint4* __restrict__ kout, uint4* __restrict__ vout, int slots)
+{
     const int u = unit_lower_bound(ut, sc_begin) + static_cast<int>(blockIdx.x);
     if (u >= unit_lower_bound(ut, sc_end)) return;
     const int kvh = blockIdx.y;
-    const int tid = threadIdx.x, lane = tid & 31;
-    if (tid < 32) {
-        int anchor;
-        int64_t s_u, e_u;
-        unit_range(ut, u, &anchor, &s_u, &e_u);
-        const int64_t W = (s_u - n_local > 0) ? s_u - n_local : 0;
-        const int n_s = static_cast<int>(n_sink < W ? n_sink : W);
-        for (int i = lane; i < n_s; i += 32) s_list[i] = i;
-        int base = n_s;
-        int cnt = sel_count[u];
-        cnt = cnt < 0 ? 0 : (cnt > k ? k : cnt);
-        const int32_t* sl = sel + static_cast<int64_t>(u) * k;
-        for (int c0 = 0; c0 < cnt; c0 += 32) {
-            const int i = c0 + lane;
-            bool valid = false;
-            int32_t tok = 0;
-            if (i < cnt) {
-                tok = sl[i];
-                valid = tok >= n_sink && tok < W && (i == 0 || tok > sl[i - 1]);
-            }
-            const uint32_t b = __ballot_sync(0xFFFFFFFFu, valid);
-            if (valid) s_list[base + __popc(b & ((1u << lane) - 1u))] = tok;
-            base += __popc(b);
-        }
-        if (lane == 0) {
-            s_n = base;
-            if (kvh == 0) count[u] = base;
-        }
-    }
-    __syncthreads();
-    const int n = s_n;
+    int n = count[u];
+    n = n < 0 ? 0 : (n > slots ? slots : n);
     const int n_pad = (n + 127) / 128 * 128;
+    const int s0 = static_cast<int>(blockIdx.z) * kPackSlots;
+    const int s1 = (s0 + kPackSlots < n_pad) ? s0 + kPackSlots : n_pad;
+    if (s0 >= s1) return;
+    const int32_t* lu = list + static_cast<int64_t>(u) * slots;
     const int64_t plane = (static_cast<int64_t>(u) * Hkv + kvh) * slots * 16;  // 16-byte chunks
     const uint4 zero = make_uint4(0, 0, 0, 0);
-    for (int i = tid; i < n_pad * 16; i += blockDim.x) {
+    for (int i = s0 * 16 + static_cast<int>(threadIdx.x); i < s1 * 16; i += blockDim.x) {
         const int slot = i >> 4, c = i & 15;
         uint4 kx = zero, vx = zero;
         if (slot < n) {
-            const int64_t src = (static_cast<int64_t>(s_list[slot]) * Hkv + kvh) * 16 + c;
+            const int64_t src = (static_cast<int64_t>(lu[slot]) * Hkv + kvh) * 16 + c;
             kx = kin[src];
             vx = vin[src];
         }
@@ -641,15 +650,14 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
     a.timeout_ns = timeout_ns;
 
     if (tok) {
-        const size_t list_bytes = static_cast<size_t>(slots) * sizeof(int32_t);
-        cudaError_t e = cudaFuncSetAttribute(k_tok_pack, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(list_bytes));
-        if (e != cudaSuccess) return e;
-        k_tok_pack<<<dim3(a.n_sc, d.Hkv), 256, list_bytes, st>>>(
-            a.ut, a.sc_begin, a.sc_end, d.n_sink, d.n_local, d.k, d.Hkv, sel_blocks, sel_count,
-            static_cast<const uint4*>(k), static_cast<const uint4*>(v),
-            reinterpret_cast<uint4*>(ws + lay.tok_pack_k), reinterpret_cast<uint4*>(ws + lay.tok_pack_v),
-            const_cast<int32_t*>(a.tok_count), slots);
+        int32_t* list = reinterpret_cast<int32_t*>(ws + lay.tok_list);
+        int32_t* cnt = const_cast<int32_t*>(a.tok_count);
+        k_tok_lists<<<a.n_sc, 32, 0, st>>>(a.ut, a.sc_begin, a.sc_end, d.n_sink, d.n_local, d.k, sel_blocks,
+                                           sel_count, list, cnt, slots);
+        k_tok_pack<<<dim3(a.n_sc, d.Hkv, (slots + kPackSlots - 1) / kPackSlots), 256, 0, st>>>(
+            a.ut, a.sc_begin, a.sc_end, d.Hkv, list, cnt, static_cast<const uint4*>(k),
+            static_cast<const uint4*>(v), reinterpret_cast<uint4*>(ws + lay.tok_pack_k),
+            reinterpret_cast<uint4*>(ws + lay.tok_pack_v), slots);
     }
     auto kern = tok ? k_sparse_attn<true> : k_sparse_attn<false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -46,6 +46,7 @@ struct WsLayout {
     size_t logits;      // fp32 [M][H_q][nb]     (block size > 1 only)
     size_t tok_split;   // bf16 [3][H_kv][M][g][128]  fingerprint parts (block size 1 only)
     size_t tok_part;    // float2 [M][H_q][ranges]    per-range softmax partials (block size 1 only)
+    size_t tok_list;    // int32 [M][slots]           distant token list of each unit (block size 1 only)
     size_t tok_pack_k;  // bf16 [M][H_kv][slots][128] distant keys of each unit, packed (block size 1 only)
     size_t tok_pack_v;  // bf16 [M][H_kv][slots][128] distant values, packed
     size_t tok_count;   // int32 [M]                  distant keys of each unit

@@ -173,45 +173,21 @@ __device__ __forceinline__ uint32_t float_key(float f)
     return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-__device__ int scan_excl(int f, int* sh, int* total)
-{
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    int x = f;
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xFFFFFFFFu, x, o);
-        if (lane >= o) x += y;
-    }
-    if (lane == 31) sh[w] = x;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int run = 0;
-        for (int i = 0; i < nw; ++i) {
-            const int t = sh[i];
-            sh[i] = run;
-            run += t;
-        }
-        sh[nw] = run;
-    }
-    __syncthreads();
-    const int r = sh[w] + x - f;
-    *total = sh[nw];
-    __syncthreads();
-    return r;
-}
-
-constexpr int kTopkThreads = 512;
+constexpr int kTopkThreads = 1024;
+constexpr int kTopkUnroll = 16;  // independent loads in flight per thread
 
 // One CTA per unit. The k-th largest key T is found with four 8-bit radix
-// passes; the selected blocks are those with key > T plus the lowest-indexed
-// ones with key == T, emitted in ascending block order: every thread owns a
-// contiguous span of candidates, counts its picks, and writes them after one
-// block-wide scan of the counts (thread order = index order).
+// passes (16 coalesced loads in flight per thread); the selected blocks are
+// those with key > T plus the lowest-indexed ones with key == T, emitted in
+// ascending block order: every warp owns a contiguous segment, counts its
+// picks, and after one scan over the warps writes them in order with
+// warp-level prefix sums.
 __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* __restrict__ scores,
                                                        int32_t* __restrict__ sel,
                                                        int32_t* __restrict__ sel_count)
 {
     __shared__ int hist[256];
-    __shared__ int sh[40];
+    __shared__ int whist[kTopkThreads / 32][256];  // per-warp histograms
     __shared__ uint32_t s_prefix;
     __shared__ int s_need;
     const int u_first = unit_lower_bound(a.ut, a.sc_begin);
@@ -236,13 +212,32 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
         s_need = a.k;
     }
     uint32_t mask = 0;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int shift = 24; shift >= 0; shift -= 8) {
-        for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+        for (int i = threadIdx.x; i < (kTopkThreads / 32) * 256; i += blockDim.x) (&whist[0][0])[i] = 0;
         __syncthreads();
         const uint32_t prefix = s_prefix;
-        for (int64_t b = lo + threadIdx.x; b < hi; b += blockDim.x) {
-            const uint32_t key = float_key(sc[b]);
-            if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+        // Every warp counts into its own histogram (keys of similar magnitude
+        // share digits, so one shared histogram would serialise on a few bins).
+        for (int64_t b0 = lo; b0 < hi; b0 += kTopkUnroll * static_cast<int64_t>(blockDim.x)) {
+            uint32_t key[kTopkUnroll];
+#pragma unroll
+            for (int j = 0; j < kTopkUnroll; ++j) {
+                const int64_t b = b0 + j * blockDim.x + threadIdx.x;
+                key[j] = b < hi ? float_key(sc[b]) : 0u;
+            }
+#pragma unroll
+            for (int j = 0; j < kTopkUnroll; ++j) {
+                const int64_t b = b0 + j * blockDim.x + threadIdx.x;
+                const bool in = b < hi && (key[j] & mask) == prefix;
+                if (in) atomicAdd(&whist[warp][(key[j] >> shift) & 255u], 1);
+            }
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < 256; i += blockDim.x) {
+            int c = 0;
+            for (int w = 0; w < kTopkThreads / 32; ++w) c += whist[w][i];
+            hist[i] = c;
         }
         __syncthreads();
         if (threadIdx.x == 0) {
@@ -259,29 +254,92 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
     }
     const uint32_t T = s_prefix;
     const int need_eq = s_need;  // how many keys equal to T to take, lowest b first
-    const int64_t span = (n + blockDim.x - 1) / blockDim.x;
-    const int64_t b0 = lo + span * threadIdx.x;
-    const int64_t b1 = (b0 + span < hi) ? b0 + span : hi;
+    // Ordered compaction: warp w owns the contiguous segment [w0, w1); lane l
+    // reads keys w0 + 128 i + 4 l .. + 3, so every step is one coalesced 512-byte
+    // read and index order within the warp is (step, lane, j).
+    const int nw = blockDim.x >> 5;
+    const int64_t seg = ((n + nw - 1) / nw + 127) / 128 * 128;
+    const int64_t w0 = lo + seg * warp;
+    const int64_t w1 = (w0 + seg < hi) ? w0 + seg : hi;
+    auto load4 = [&](int64_t b, uint32_t (&key)[4]) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) key[j] = (b + j < w1) ? float_key(sc[b + j]) : 0u;
+    };
     int n_gt = 0, n_eq = 0;
-    for (int64_t b = b0; b < b1; ++b) {
-        const uint32_t key = float_key(sc[b]);
-        n_gt += key > T;
-        n_eq += key == T;
-    }
-    int total;
-    const int eq_before = scan_excl(n_eq, sh, &total);
-    int take_eq = need_eq - eq_before;
-    take_eq = take_eq < 0 ? 0 : (take_eq > n_eq ? n_eq : take_eq);
-    int taken;
-    int pos = scan_excl(n_gt + take_eq, sh, &taken);
-    for (int64_t b = b0; b < b1; ++b) {
-        const uint32_t key = float_key(sc[b]);
-        if (key > T) {
-            out[pos++] = static_cast<int32_t>(b);
-        } else if (key == T && take_eq > 0) {
-            out[pos++] = static_cast<int32_t>(b);
-            --take_eq;
+    for (int64_t b = w0 + 4 * lane; b < w1; b += 128) {
+        uint32_t key[4];
+        load4(b, key);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            n_gt += (b + j < w1) && key[j] > T;
+            n_eq += (b + j < w1) && key[j] == T;
         }
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        n_gt += __shfl_xor_sync(0xFFFFFFFFu, n_gt, o);
+        n_eq += __shfl_xor_sync(0xFFFFFFFFu, n_eq, o);
+    }
+    __shared__ int s_take[kTopkThreads / 32], s_pos[kTopkThreads / 32], s_taken;
+    if (lane == 0) {
+        s_take[warp] = n_eq;  // equal keys of this warp, for now
+        s_pos[warp] = n_gt;   // keys above T of this warp, for now
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int eq_before = 0, pos = 0;
+        for (int w = 0; w < nw; ++w) {
+            const int e = s_take[w], g = s_pos[w];
+            int take = need_eq - eq_before;
+            take = take < 0 ? 0 : (take > e ? e : take);
+            eq_before += e;
+            s_take[w] = take;
+            s_pos[w] = pos;
+            pos += g + take;
+        }
+        s_taken = pos;
+    }
+    __syncthreads();
+    const int taken = s_taken;
+    int pos = s_pos[warp], take_eq = s_take[warp];
+    for (int64_t b = w0 + 4 * lane; b < w1; b += 128) {
+        uint32_t key[4];
+        load4(b, key);
+        int gt_l = 0, eq_l = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            gt_l += (b + j < w1) && key[j] > T;
+            eq_l += (b + j < w1) && key[j] == T;
+        }
+        // exclusive prefix over lanes of the equal keys
+        int eq_inc = eq_l;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, eq_inc, o);
+            if (lane >= o) eq_inc += y;
+        }
+        const int eq_tot = __shfl_sync(0xFFFFFFFFu, eq_inc, 31);
+        int eq_rank = eq_inc - eq_l;  // equal keys before this lane in this step
+        // picks of this lane: keys above T and the equal keys still to take
+        int pk[4], n_pk = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            pk[j] = 0;
+            if (b + j < w1) {
+                if (key[j] > T) pk[j] = 1;
+                else if (key[j] == T) pk[j] = (eq_rank++ < take_eq);
+            }
+            n_pk += pk[j];
+        }
+        int pk_inc = n_pk;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, pk_inc, o);
+            if (lane >= o) pk_inc += y;
+        }
+        int p = pos + pk_inc - n_pk;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (pk[j]) out[p++] = static_cast<int32_t>(b + j);
+        pos += __shfl_sync(0xFFFFFFFFu, pk_inc, 31);
+        take_eq -= (eq_tot < take_eq ? eq_tot : take_eq);
     }
     for (int i = taken + threadIdx.x; i < a.k; i += blockDim.x) out[i] = -1;
     if (threadIdx.x == 0) sel_count[u] = taken;

@@ -364,12 +364,15 @@ __global__ void __launch_bounds__(128) k_tok_split(TokArgs a, const float* __res
     parts[2 * plane + off] = v3;
 }
 
-// One thread per (unit, head): merge the token ranges' (max, sum) in order.
+// One warp per (unit, head): merge the token ranges' (max, sum); the lanes
+// take ranges in a fixed interleave and combine in a fixed tree, so the result
+// does not depend on scheduling.
 __global__ void __launch_bounds__(256) k_tok_merge(TokArgs a)
 {
     const int u_first = unit_lower_bound(a.ut, a.sc_begin);
     const int u_end = unit_lower_bound(a.ut, a.sc_end);
-    const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    const int64_t i = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
     const int u = u_first + static_cast<int>(i / a.Hq);
     const int h = static_cast<int>(i % a.Hq);
     if (u >= u_end) return;
@@ -379,12 +382,15 @@ __global__ void __launch_bounds__(256) k_tok_merge(TokArgs a)
     if (hi > a.n_sink) {
         const float2* pr = a.part + (static_cast<int64_t>(u) * a.Hq + h) * a.n_ranges;
         const int x0 = a.n_sink / a.range, x1 = (hi + a.range - 1) / a.range;
-        for (int xx = x0; xx < x1; ++xx) m = fmaxf(m, pr[xx].x);
-        for (int xx = x0; xx < x1; ++xx)
+        for (int xx = x0 + lane; xx < x1; xx += 32) m = fmaxf(m, pr[xx].x);
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+        for (int xx = x0 + lane; xx < x1; xx += 32)
             if (pr[xx].x > -INFINITY) sum += pr[xx].y * ex2(pr[xx].x - m);
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
     }
-    const_cast<float2*>(a.stats)[static_cast<int64_t>(u) * a.Hq + h] =
-        make_float2(m, sum > 0.f ? 1.0f / sum : 0.f);
+    if (lane == 0)
+        const_cast<float2*>(a.stats)[static_cast<int64_t>(u) * a.Hq + h] =
+            make_float2(m, sum > 0.f ? 1.0f / sum : 0.f);
 }
 
 template <int G>
@@ -402,7 +408,7 @@ cudaError_t run_tok_passes(dim3 grid, int64_t rows, const CUtensorMap& tf, const
         attr = true;
     }
     k_tok_score<0, G><<<grid, kTokThreads, kSmemTok0, st>>>(tf, tk, a);
-    k_tok_merge<<<static_cast<unsigned>((rows + 255) / 256), 256, 0, st>>>(a);
+    k_tok_merge<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a);
     k_tok_score<1, G><<<grid, kTokThreads, kSmemTok1, st>>>(tf, tk, a);
     return cudaGetLastError();
 }
