@@ -49,6 +49,8 @@ def parse_args():
                     help="skip timing the per-sub-chunk selection mode alongside")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle sample")
+    ap.add_argument("--paged", type=int, default=0, metavar="P",
+                    help="keep K and V in a paged cache of P-token pages (shuffled page order)")
     ap.add_argument("--sweep", action="store_true",
                     help="clustering-threshold sweep (theta x L_max) on planted-topic data: cluster sizes, "
                          "overlap ratio rho, boundary recall and step time (one JSON line)")
@@ -277,6 +279,21 @@ def run_scale(args):
     p = S.params_for(w)
     buf = pkg.allocate(p, mode)
     stream = torch.cuda.current_stream()
+    kv = None
+    if args.paged:
+        # K and V moved into a pool of pages in shuffled order (plus spare pages)
+        P = args.paged
+        n_pages = -(-w.n_tokens // P)
+        order = torch.from_numpy(np.random.default_rng(1).permutation(n_pages + 4)[:n_pages].astype(np.int32)).cuda()
+        pools = []
+        for x in dev[1:]:
+            pool = torch.zeros((n_pages + 4, P, w.num_kv_heads, w.head_dim), dtype=x.dtype, device="cuda")
+            full = torch.zeros((n_pages * P, w.num_kv_heads, w.head_dim), dtype=x.dtype, device="cuda")
+            full[: w.n_tokens] = x
+            pool[order.long()] = full.view(n_pages, P, w.num_kv_heads, w.head_dim)
+            pools.append(pool)
+            del full
+        kv = S.kv_pages(pools[0], pools[1], order, P)
 
     def barrier():
         if world > 1:
@@ -296,13 +313,27 @@ def run_scale(args):
         for i in range(steps):
             e = ev[i]
             e[0].record(stream)
-            S.scale_build_reps(p, dev[0], dev[1], buf_.reps, buf_.fingerprints, buf_.unit_start,
-                               buf_.n_units, buf_.ws, stream)
+            if kv is not None:
+                S.scale_build_reps_paged(p, dev[0], kv, buf_.reps, buf_.fingerprints, buf_.unit_start,
+                                         buf_.n_units, buf_.ws, stream)
+            else:
+                S.scale_build_reps(p, dev[0], dev[1], buf_.reps, buf_.fingerprints, buf_.unit_start,
+                                   buf_.n_units, buf_.ws, stream)
             e[1].record(stream)
-            S.select(p, mode_, 0, w.n_tokens, dev[1], buf_, stream)
+            if kv is not None and w.block_size == 1:
+                S.scale_select_tokens_paged(p, mode_, 0, w.n_tokens, kv, buf_.fingerprints, buf_.unit_start,
+                                            buf_.n_units, buf_.sel_blocks, buf_.sel_count, None, buf_.ws,
+                                            stream)
+            else:
+                S.select(p, mode_, 0, w.n_tokens, dev[1], buf_, stream)
             e[2].record(stream)
-            S.scale_sparse_prefill(p, mode_, 0, w.n_tokens, *dev, buf_.unit_start, buf_.n_units,
-                                   buf_.sel_blocks, buf_.sel_count, buf_.out, buf_.ws, stream)
+            if kv is not None:
+                S.scale_sparse_prefill_paged(p, mode_, 0, w.n_tokens, dev[0], kv, buf_.unit_start,
+                                             buf_.n_units, buf_.sel_blocks, buf_.sel_count, buf_.out,
+                                             buf_.ws, stream)
+            else:
+                S.scale_sparse_prefill(p, mode_, 0, w.n_tokens, *dev, buf_.unit_start, buf_.n_units,
+                                       buf_.sel_blocks, buf_.sel_count, buf_.out, buf_.ws, stream)
             e[3].record(stream)
         end.record(stream)
         torch.cuda.synchronize()
@@ -351,6 +382,7 @@ def run_scale(args):
                    "max_cluster_subchunks": w.max_cluster_subchunks, "block_size": w.block_size,
                    "top_k": w.top_k, "n_sink": w.n_sink, "n_local": w.n_local, "theta": w.theta,
                    "mode": args.mode, "parallelism": f"independent layers x{world}",
+                   "kv_layout": f"paged, {args.paged}-token pages" if args.paged else "contiguous",
                    "l2": "inputs larger than L2 (Q+K+V %.2f GB)" % ((q.nbytes + k.nbytes + v.nbytes) / 1e9)},
         "stages_ms": {"build_reps": stages[0], "select": stages[1], "sparse_attention": stages[2]},
         "retrieval_calls": calls,

@@ -203,6 +203,50 @@ int scale_sparse_prefill(const scale_params_t *p, int32_t mode, int64_t tok_begi
                          const int32_t *sel_blocks, const int32_t *sel_count, void *out,
                          void *ws, size_t ws_bytes, scale_stream_t stream);
 
+/* Paged KV cache (the serving layout, as paged attention engines keep it):
+ * K and V live in a pool of num_pages pages of page_size tokens,
+ *   k_pages, v_pages  bf16 [num_pages][page_size][H_kv][128]  (device)
+ * and token t of the sequence is row t % page_size of page
+ * page_table[t / page_size] (int32, device, ceil(N / page_size) entries).
+ * The *_paged entry points below compute exactly what their contiguous
+ * counterparts compute (bit for bit, for the same K and V values).
+ *  - Every K/V box the kernels load is 64 rows starting at a multiple of 64,
+ *    so page_size, sub_chunk, n_sink and n_local must be multiples of 64 and
+ *    block_size 1 or a multiple of 64 (SCALE_ERR_UNSUPPORTED otherwise), and
+ *    num_pages * page_size < 2^31.
+ *  - A page-table entry outside [0, num_pages) is not dereferenced: its
+ *    tokens read as zero keys and values. Q and the attention output stay
+ *    contiguous.
+ *  - The rows of the last page past token N - 1 are loaded with their box and
+ *    masked out (weight exactly 0); they must hold finite values (zeros, or
+ *    any data), since 0 times a NaN would still be NaN. */
+typedef struct {
+    const void *k_pages;
+    const void *v_pages;
+    const int32_t *page_table;
+    int32_t page_size;
+    int64_t num_pages;
+} scale_kv_pages_t;
+
+/* scale_build_reps with K read from a paged cache. */
+int scale_build_reps_paged(const scale_params_t *p, const void *q, const scale_kv_pages_t *kv,
+                           float *reps, float *fingerprints, int32_t *unit_start, int32_t *n_units,
+                           void *ws, size_t ws_bytes, scale_stream_t stream);
+
+/* scale_select_tokens with K read from a paged cache. */
+int scale_select_tokens_paged(const scale_params_t *p, int32_t mode, int64_t tok_begin,
+                              int64_t tok_end, const scale_kv_pages_t *kv, const float *fingerprints,
+                              const int32_t *unit_start, const int32_t *n_units, int32_t *sel_tokens,
+                              int32_t *sel_count, float *sel_scores, void *ws, size_t ws_bytes,
+                              scale_stream_t stream);
+
+/* scale_sparse_prefill with K and V read from a paged cache. */
+int scale_sparse_prefill_paged(const scale_params_t *p, int32_t mode, int64_t tok_begin,
+                               int64_t tok_end, const void *q, const scale_kv_pages_t *kv,
+                               const int32_t *unit_start, const int32_t *n_units,
+                               const int32_t *sel_blocks, const int32_t *sel_count, void *out,
+                               void *ws, size_t ws_bytes, scale_stream_t stream);
+
 /* Synchronous: waits for `stream`, then reads the device status word of `ws`
  * into *status (SCALE_OK, SCALE_ERR_TIMEOUT or SCALE_ERR_DEVICE). The word is
  * sticky until scale_workspace_init(). */

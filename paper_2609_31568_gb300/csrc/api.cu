@@ -116,6 +116,23 @@ int check_range(const Derived& d, int mode, int64_t tb, int64_t te)
 
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? SCALE_OK : SCALE_ERR_CUDA; }
 
+KvPaging contiguous(const Derived& d) { return KvPaging{nullptr, 0, 0, d.N, d.N}; }
+
+// A page pool that the kernels can read: every box they load is 64 rows
+// starting at a multiple of 64, so page sizes, sub-chunks, sinks, windows and
+// blocks must be multiples of 64 (blocks may also be single tokens).
+int check_pages(const Derived& d, const scale_kv_pages_t* kv, KvPaging* pg)
+{
+    if (!kv || kv->page_size <= 0 || kv->num_pages <= 0) return SCALE_ERR_INVALID_ARG;
+    if (kv->page_size % 64 || d.L % 64 || d.n_sink % 64 || d.n_local % 64 || (d.B != 1 && d.B % 64))
+        return SCALE_ERR_UNSUPPORTED;
+    if (kv->num_pages * kv->page_size >= (1ll << 31) - 256) return SCALE_ERR_UNSUPPORTED;
+    if (!device_ptr(kv->k_pages, 16) || !device_ptr(kv->v_pages, 16) || !device_ptr(kv->page_table, 4))
+        return SCALE_ERR_INVALID_ARG;
+    *pg = KvPaging{kv->page_table, kv->page_size, kv->num_pages, d.N, kv->num_pages * kv->page_size};
+    return SCALE_OK;
+}
+
 struct Arena {
     size_t q, k, v, out, reps, fp, unit_start, n_units, sel, sel_count, ws, total;
 };
@@ -185,6 +202,19 @@ int scale_workspace_init(void* ws, size_t ws_bytes, scale_stream_t stream)
     return cuda_status(cudaMemsetAsync(ws, 0, 256, stream));
 }
 
+static int build_reps_impl(const Derived& d, const void* q, const void* k, const KvPaging& pg,
+                           float* reps, float* fingerprints, int32_t* unit_start, int32_t* n_units,
+                           void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    int rc;
+    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !(device_ptr(reps, 16) || (!reps && d.B == 1)) ||
+        !device_ptr(fingerprints, 16) || !device_ptr(unit_start, 4) || !device_ptr(n_units, 4))
+        return SCALE_ERR_INVALID_ARG;
+    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
+    return cuda_status(launch_build_reps(d, q, k, pg, reps, fingerprints, unit_start, n_units,
+                                         static_cast<uint8_t*>(ws), stream));
+}
+
 int scale_build_reps(const scale_params_t* p, const void* q, const void* k, float* reps,
                      float* fingerprints, int32_t* unit_start, int32_t* n_units, void* ws,
                      size_t ws_bytes, scale_stream_t stream)
@@ -192,12 +222,21 @@ int scale_build_reps(const scale_params_t* p, const void* q, const void* k, floa
     Derived d;
     int rc = derive(p, &d);
     if (rc) return rc;
-    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !(device_ptr(reps, 16) || (!reps && d.B == 1)) ||
-        !device_ptr(fingerprints, 16) || !device_ptr(unit_start, 4) || !device_ptr(n_units, 4))
-        return SCALE_ERR_INVALID_ARG;
-    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
-    return cuda_status(launch_build_reps(d, q, k, reps, fingerprints, unit_start, n_units,
-                                         static_cast<uint8_t*>(ws), stream));
+    return build_reps_impl(d, q, k, contiguous(d), reps, fingerprints, unit_start, n_units, ws, ws_bytes,
+                           stream);
+}
+
+int scale_build_reps_paged(const scale_params_t* p, const void* q, const scale_kv_pages_t* kv, float* reps,
+                           float* fingerprints, int32_t* unit_start, int32_t* n_units, void* ws,
+                           size_t ws_bytes, scale_stream_t stream)
+{
+    Derived d;
+    KvPaging pg;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if ((rc = check_pages(d, kv, &pg))) return rc;
+    return build_reps_impl(d, q, kv->k_pages, pg, reps, fingerprints, unit_start, n_units, ws, ws_bytes,
+                           stream);
 }
 
 int scale_select(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
@@ -222,14 +261,13 @@ int scale_select(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64
                                      static_cast<uint8_t*>(ws), stream));
 }
 
-int scale_select_tokens(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
-                        const void* k, const float* fingerprints, const int32_t* unit_start,
-                        const int32_t* n_units, int32_t* sel_tokens, int32_t* sel_count,
-                        float* sel_scores, void* ws, size_t ws_bytes, scale_stream_t stream)
+static int select_tokens_impl(const Derived& d, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                              const void* k, const KvPaging& pg, const float* fingerprints,
+                              const int32_t* unit_start, const int32_t* n_units, int32_t* sel_tokens,
+                              int32_t* sel_count, float* sel_scores, void* ws, size_t ws_bytes,
+                              scale_stream_t stream)
 {
-    Derived d;
-    int rc = derive(p, &d);
-    if (rc) return rc;
+    int rc;
     if (d.B != 1) return SCALE_ERR_INVALID_ARG;
     if (d.g != 1 && d.g != 2 && d.g != 4 && d.g != 8) return SCALE_ERR_UNSUPPORTED;
     if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
@@ -240,9 +278,59 @@ int scale_select_tokens(const scale_params_t* p, int32_t mode, int64_t tok_begin
         return SCALE_ERR_INVALID_ARG;
     if ((rc = check_ws(d, ws, ws_bytes))) return rc;
     if (tok_begin == tok_end) return SCALE_OK;
-    return cuda_status(launch_select_tokens(d, mode, tok_begin, tok_end, k, fingerprints, unit_start,
+    return cuda_status(launch_select_tokens(d, mode, tok_begin, tok_end, k, pg, fingerprints, unit_start,
                                             n_units, sel_tokens, sel_count, sel_scores,
                                             static_cast<uint8_t*>(ws), g_timeout_ns.load(), stream));
+}
+
+int scale_select_tokens(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                        const void* k, const float* fingerprints, const int32_t* unit_start,
+                        const int32_t* n_units, int32_t* sel_tokens, int32_t* sel_count,
+                        float* sel_scores, void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    return select_tokens_impl(d, mode, tok_begin, tok_end, k, contiguous(d), fingerprints, unit_start,
+                              n_units, sel_tokens, sel_count, sel_scores, ws, ws_bytes, stream);
+}
+
+int scale_select_tokens_paged(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                              const scale_kv_pages_t* kv, const float* fingerprints,
+                              const int32_t* unit_start, const int32_t* n_units, int32_t* sel_tokens,
+                              int32_t* sel_count, float* sel_scores, void* ws, size_t ws_bytes,
+                              scale_stream_t stream)
+{
+    Derived d;
+    KvPaging pg;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (d.B != 1) return SCALE_ERR_INVALID_ARG;
+    if ((rc = check_pages(d, kv, &pg))) return rc;
+    return select_tokens_impl(d, mode, tok_begin, tok_end, kv->k_pages, pg, fingerprints, unit_start,
+                              n_units, sel_tokens, sel_count, sel_scores, ws, ws_bytes, stream);
+}
+
+static int sparse_prefill_impl(const Derived& d, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                               const void* q, const void* k, const void* v, const KvPaging& pg,
+                               const int32_t* unit_start, const int32_t* n_units,
+                               const int32_t* sel_blocks, const int32_t* sel_count, void* out, void* ws,
+                               size_t ws_bytes, scale_stream_t stream)
+{
+    int rc;
+    if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
+    if (d.g % 2) return SCALE_ERR_UNSUPPORTED;
+    if (d.B > 1 && max_distant_segments(d) > kMaxSegments) return SCALE_ERR_UNSUPPORTED;
+    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(v, 16) || !device_ptr(out, 16) ||
+        !device_ptr(sel_count, 4) || (d.k > 0 && !device_ptr(sel_blocks, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if (mode == SCALE_MODE_PER_CLUSTER && (!device_ptr(unit_start, 4) || !device_ptr(n_units, 4)))
+        return SCALE_ERR_INVALID_ARG;
+    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
+    if (tok_begin == tok_end) return SCALE_OK;
+    return cuda_status(launch_sparse_prefill(d, mode, tok_begin, tok_end, q, k, v, pg, unit_start,
+                                             n_units, sel_blocks, sel_count, out,
+                                             static_cast<uint8_t*>(ws), g_timeout_ns.load(), stream));
 }
 
 int scale_sparse_prefill(const scale_params_t* p, int32_t mode, int64_t tok_begin,
@@ -254,20 +342,23 @@ int scale_sparse_prefill(const scale_params_t* p, int32_t mode, int64_t tok_begi
     Derived d;
     int rc = derive(p, &d);
     if (rc) return rc;
-    if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
-    if (d.g % 2) return SCALE_ERR_UNSUPPORTED;
-    if (d.B > 1 && max_distant_segments(d) > kMaxSegments) return SCALE_ERR_UNSUPPORTED;
-    if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(v, 16) || !device_ptr(out, 16) ||
-        !device_ptr(sel_count, 4) || (d.k > 0 && !device_ptr(sel_blocks, 4)))
-        return SCALE_ERR_INVALID_ARG;
-    if (mode == SCALE_MODE_PER_CLUSTER && (!device_ptr(unit_start, 4) || !device_ptr(n_units, 4)))
-        return SCALE_ERR_INVALID_ARG;
-    if ((rc = check_ws(d, ws, ws_bytes))) return rc;
-    if (tok_begin == tok_end) return SCALE_OK;
-    return cuda_status(launch_sparse_prefill(d, mode, tok_begin, tok_end, q, k, v, unit_start,
-                                             n_units, sel_blocks, sel_count, out,
-                                             static_cast<uint8_t*>(ws), g_timeout_ns.load(),
-                                             stream));
+    return sparse_prefill_impl(d, mode, tok_begin, tok_end, q, k, v, contiguous(d), unit_start, n_units,
+                               sel_blocks, sel_count, out, ws, ws_bytes, stream);
+}
+
+int scale_sparse_prefill_paged(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
+                               const void* q, const scale_kv_pages_t* kv, const int32_t* unit_start,
+                               const int32_t* n_units, const int32_t* sel_blocks,
+                               const int32_t* sel_count, void* out, void* ws, size_t ws_bytes,
+                               scale_stream_t stream)
+{
+    Derived d;
+    KvPaging pg;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if ((rc = check_pages(d, kv, &pg))) return rc;
+    return sparse_prefill_impl(d, mode, tok_begin, tok_end, q, kv->k_pages, kv->v_pages, pg, unit_start,
+                               n_units, sel_blocks, sel_count, out, ws, ws_bytes, stream);
 }
 
 int scale_get_device_status(const void* ws, scale_stream_t stream, int32_t* status)

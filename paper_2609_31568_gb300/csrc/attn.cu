@@ -75,6 +75,7 @@ struct AttnArgs {
     __nv_bfloat16* out;
     int32_t* status;
     uint64_t timeout_ns;
+    KvPaging pg;
 };
 
 struct Barriers {
@@ -257,6 +258,9 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                     ta = static_cast<int32_t>(W + 128ll * (t - n_dt));
                     tb = ta + 64;
                 }
+                // 64-row boxes: every one lies inside one KV page
+                const int32_t ra = packed ? 0 : kv_row_tma(a.pg, ta);
+                const int32_t rb = packed ? 0 : kv_row_tma(a.pg, tb);
                 if (t >= 2 && !mbar_wait_bounded(&bars.k_empty[st], ph, a.timeout_ns, &abort_flag)) {
                     fail(&abort_flag, a.status);
                     break;
@@ -268,8 +272,8 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                     if (packed) {
                         tma_load_3d(kd + hf * kHalf, &tpk, &bars.k_full[st], hf * 64, ta, prow);
                     } else {
-                        tma_load_3d(kd + hf * kHalf, &tk, &bars.k_full[st], hf * 64, kvh, ta);
-                        tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.k_full[st], hf * 64, kvh, tb);
+                        tma_load_3d(kd + hf * kHalf, &tk, &bars.k_full[st], hf * 64, kvh, ra);
+                        tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.k_full[st], hf * 64, kvh, rb);
                     }
                 }
                 if (t >= 2 && !mbar_wait_bounded(&bars.v_empty[st], ph, a.timeout_ns, &abort_flag)) {
@@ -283,8 +287,8 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                     if (packed) {
                         tma_load_3d(vd + hf * kHalf, &tpv, &bars.v_full[st], hf * 64, ta, prow);
                     } else {
-                        tma_load_3d(vd + hf * kHalf, &tv, &bars.v_full[st], hf * 64, kvh, ta);
-                        tma_load_3d(vd + hf * kHalf + kSegBytes, &tv, &bars.v_full[st], hf * 64, kvh, tb);
+                        tma_load_3d(vd + hf * kHalf, &tv, &bars.v_full[st], hf * 64, kvh, ra);
+                        tma_load_3d(vd + hf * kHalf + kSegBytes, &tv, &bars.v_full[st], hf * 64, kvh, rb);
                     }
                 }
             }
@@ -536,7 +540,7 @@ __global__ void __launch_bounds__(32) k_tok_lists(Units ut, int sc_begin, int sc
 // z = blockIdx.z, into contiguous rows [M * H_kv][slots][128]; slots past the
 // list up to the next multiple of 128 are written as zeros.
 constexpr int kPackSlots = 256;
-__global__ void __launch_bounds__(256) k_tok_pack(Units ut, int sc_begin, int sc_end, int Hkv,
+__global__ void __launch_bounds__(256) k_tok_pack(Units ut, int sc_begin, int sc_end, int Hkv, KvPaging pg,
                                                   const int32_t* __restrict__ list,
                                                   const int32_t* __restrict__ count,
                                                   const uint4* __restrict__ kin, const uint4* __restrict__ vin,
@@ -557,8 +561,9 @@ __global__ void __launch_bounds__(256) k_tok_pack(Units ut, int sc_begin, int sc
     for (int i = s0 * 16 + static_cast<int>(threadIdx.x); i < s1 * 16; i += blockDim.x) {
         const int slot = i >> 4, c = i & 15;
         uint4 kx = zero, vx = zero;
-        if (slot < n) {
-            const int64_t src = (static_cast<int64_t>(lu[slot]) * Hkv + kvh) * 16 + c;
+        const int64_t row = slot < n ? kv_row(pg, lu[slot]) : -1;  // -1: zeros
+        if (row >= 0) {
+            const int64_t src = (row * Hkv + kvh) * 16 + c;
             kx = kin[src];
             vx = vin[src];
         }
@@ -597,15 +602,15 @@ int64_t max_distant_segments(const Derived& d)
 }
 
 cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
-                                  const void* q, const void* k, const void* v,
+                                  const void* q, const void* k, const void* v, const KvPaging& pg,
                                   const int32_t* unit_start, const int32_t* n_units,
                                   const int32_t* sel_blocks, const int32_t* sel_count, void* out,
                                   uint8_t* ws, uint64_t timeout_ns, cudaStream_t st)
 {
     CUtensorMap tq, tk, tv, tpk, tpv;
     if (!scale_host::make_token_major_map(&tq, q, kHeadDim, d.Hq, d.N, 64, 128) ||
-        !scale_host::make_token_major_map(&tk, k, kHeadDim, d.Hkv, d.N, 64, 64) ||
-        !scale_host::make_token_major_map(&tv, v, kHeadDim, d.Hkv, d.N, 64, 64))
+        !scale_host::make_token_major_map(&tk, k, kHeadDim, d.Hkv, pg.page_table ? pg.pool_rows : d.N, 64, 64) ||
+        !scale_host::make_token_major_map(&tv, v, kHeadDim, d.Hkv, pg.page_table ? pg.pool_rows : d.N, 64, 64))
         return cudaErrorInvalidValue;
     const bool tok = d.B == 1;
     const WsLayout lay = ws_layout(d);
@@ -648,6 +653,7 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
     a.out = static_cast<__nv_bfloat16*>(out);
     a.status = reinterpret_cast<int32_t*>(ws + kStatusOffset);
     a.timeout_ns = timeout_ns;
+    a.pg = pg;
 
     if (tok) {
         int32_t* list = reinterpret_cast<int32_t*>(ws + lay.tok_list);
@@ -655,7 +661,7 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
         k_tok_lists<<<a.n_sc, 32, 0, st>>>(a.ut, a.sc_begin, a.sc_end, d.n_sink, d.n_local, d.k, sel_blocks,
                                            sel_count, list, cnt, slots);
         k_tok_pack<<<dim3(a.n_sc, d.Hkv, (slots + kPackSlots - 1) / kPackSlots), 256, 0, st>>>(
-            a.ut, a.sc_begin, a.sc_end, d.Hkv, list, cnt, static_cast<const uint4*>(k),
+            a.ut, a.sc_begin, a.sc_end, d.Hkv, pg, list, cnt, static_cast<const uint4*>(k),
             static_cast<const uint4*>(v), reinterpret_cast<uint4*>(ws + lay.tok_pack_k),
             reinterpret_cast<uint4*>(ws + lay.tok_pack_v), slots);
     }

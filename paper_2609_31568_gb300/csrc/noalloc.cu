@@ -80,7 +80,8 @@ extern "C" int scale_build_reps_noalloc(const scale_params_t* p, const void* q, 
     // cleared so that it never reports an earlier call's state.
     if (cudaMemsetAsync(static_cast<uint8_t*>(scratch) + kStatusOffset, 0, 256, stream) != cudaSuccess)
         return SCALE_ERR_CUDA;
-    return launch_build_reps(d, q, k, reps, fingerprints, unit_start, n_units,
+    const KvPaging pg{nullptr, 0, 0, d.N, d.N};
+    return launch_build_reps(d, q, k, pg, reps, fingerprints, unit_start, n_units,
                              static_cast<uint8_t*>(scratch), stream) == cudaSuccess
                ? SCALE_OK
                : SCALE_ERR_CUDA;

@@ -33,7 +33,7 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p)
 // Representative key of block b for every KV head: the mean of the block's
 // keys. One CTA per block; thread c owns elements [8c, 8c+8) of the token row
 // (H_kv * 128 elements), so every token row is read as one coalesced span.
-__global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k, int64_t N,
+__global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k, KvPaging pg, int64_t N,
                                                       int row_chunks, int B, int64_t nb,
                                                       float* __restrict__ reps)
 {
@@ -43,16 +43,23 @@ __global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k
     const int64_t t0 = b * B;
     const int64_t t1 = (t0 + B < N) ? t0 + B : N;
     float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    const uint4* src = k + t0 * row_chunks + c;
+    const uint4* src = k + c;
+    const uint4 zero = make_uint4(0, 0, 0, 0);
     int64_t t = t0;
     for (; t + 8 <= t1; t += 8) {
         uint4 x[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) x[i] = ld_stream(src + (t - t0 + i) * row_chunks);
+        for (int i = 0; i < 8; ++i) {
+            const int64_t r = kv_row(pg, t + i);  // -1: a page outside the pool reads as zeros
+            x[i] = r < 0 ? zero : ld_stream(src + r * row_chunks);
+        }
 #pragma unroll
         for (int i = 0; i < 8; ++i) add_bf16x8(acc, x[i]);
     }
-    for (; t < t1; ++t) add_bf16x8(acc, ld_stream(src + (t - t0) * row_chunks));
+    for (; t < t1; ++t) {
+        const int64_t r = kv_row(pg, t);
+        add_bf16x8(acc, r < 0 ? zero : ld_stream(src + r * row_chunks));
+    }
     const float cnt = static_cast<float>(t1 - t0);
     const int j = c / (kHeadDim / 8);
     const int d0 = (c % (kHeadDim / 8)) * 8;
@@ -229,8 +236,8 @@ __global__ void __launch_bounds__(1024) k_cluster(const float* __restrict__ gram
 
 }  // namespace
 
-cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, float* reps,
-                              float* fingerprints, int32_t* unit_start, int32_t* n_units,
+cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, const KvPaging& pg,
+                              float* reps, float* fingerprints, int32_t* unit_start, int32_t* n_units,
                               uint8_t* ws, cudaStream_t st)
 {
     const WsLayout lay = ws_layout(d);
@@ -242,7 +249,7 @@ cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, fl
     const int row_chunks = d.Hkv * (kHeadDim / 8);
     if (reps)  // block size 1 may skip them: token-level selection reads K itself
         k_block_reps<<<static_cast<unsigned>(d.nb), row_chunks, 0, st>>>(
-            static_cast<const uint4*>(k), d.N, row_chunks, d.B, d.nb, reps);
+            static_cast<const uint4*>(k), pg, d.N, row_chunks, d.B, d.nb, reps);
 
     const int D8 = d.D / 8;
     const int split_len = (d.L + d.fp_splits - 1) / d.fp_splits;

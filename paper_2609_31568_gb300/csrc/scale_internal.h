@@ -113,21 +113,51 @@ __device__ __forceinline__ void unit_range(const Units& t, int u, int* anchor, i
     *e = ee < t.N ? ee : t.N;
 }
 
+// Where token t's K and V rows live: row t of contiguous [N][H_kv][128]
+// tensors (page_table == nullptr), or row page_table[t / page_size] *
+// page_size + t % page_size of a page pool [num_pages * page_size][H_kv][128].
+struct KvPaging {
+    const int32_t* page_table;
+    int page_size;
+    int64_t num_pages;
+    int64_t N;
+    int64_t pool_rows;  // rows of the pool (N when contiguous)
+};
+
+// Row of token t, or -1 for t >= N or a page-table entry outside the pool.
+__device__ __forceinline__ int64_t kv_row(const KvPaging& pg, int64_t t)
+{
+    if (t >= pg.N) return -1;
+    if (!pg.page_table) return t;
+    const int64_t lp = t / pg.page_size;
+    const int64_t page = pg.page_table[lp];
+    if (page < 0 || page >= pg.num_pages) return -1;
+    return page * pg.page_size + (t - lp * pg.page_size);
+}
+
+// TMA coordinate of token t's row: rows that do not exist map past the end of
+// the tensor, where TMA fills zeros.
+__device__ __forceinline__ int32_t kv_row_tma(const KvPaging& pg, int64_t t)
+{
+    const int64_t r = kv_row(pg, t);
+    return static_cast<int32_t>(r < 0 ? pg.pool_rows : r);
+}
+
 __device__ __forceinline__ void record_status(int32_t* status, int32_t code)
 {
     atomicCAS(status, 0, code);
 }
 
 // ---- launchers (defined in the .cu files) ----
-cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, float* reps,
-                              float* fingerprints, int32_t* unit_start, int32_t* n_units,
+cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, const KvPaging& pg,
+                              float* reps, float* fingerprints, int32_t* unit_start, int32_t* n_units,
                               uint8_t* ws, cudaStream_t st);
 cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
                           const float* reps, const float* fingerprints, const int32_t* unit_start,
                           const int32_t* n_units, int32_t* sel_blocks, int32_t* sel_count,
                           float* sel_scores, uint8_t* ws, cudaStream_t st);
 cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
-                                  const void* q, const void* k, const void* v,
+                                  const void* q, const void* k, const void* v, const KvPaging& pg,
                                   const int32_t* unit_start, const int32_t* n_units,
                                   const int32_t* sel_blocks, const int32_t* sel_count, void* out,
                                   uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
@@ -135,7 +165,8 @@ cudaError_t launch_wait_selftest(uint8_t* ws, uint64_t timeout_ns, cudaStream_t 
 cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_end, const float* scores,
                         int32_t* sel, int32_t* sel_count, cudaStream_t st);
 cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
-                                 const void* k, const float* fingerprints, const int32_t* unit_start,
+                                 const void* k, const KvPaging& pg, const float* fingerprints,
+                                 const int32_t* unit_start,
                                  const int32_t* n_units, int32_t* sel, int32_t* sel_count,
                                  float* sel_scores, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 // Tokens per CTA of the token-level scoring kernels.

@@ -64,6 +64,7 @@ struct TokArgs {
     float* scores;      // [M][N]
     int32_t* status;
     uint64_t timeout_ns;
+    KvPaging pg;
 };
 
 struct TokBars {
@@ -176,9 +177,14 @@ k_tok_score(const __grid_constant__ CUtensorMap tf, const __grid_constant__ CUte
                     }
                     mbar_arrive_expect_tx(&bars.k_full[st], kTile);
                     if (st) ++issued_k1; else ++issued_k0;
-                    for (int hf = 0; hf < 2; ++hf)
-                        tma_load_3d(smem + kOffK + st * kTile + hf * kHalfT, &tk, &bars.k_full[st], hf * 64, j,
-                                    r0 + 128 * i);
+                    // two 64-row boxes per half: each lies inside one KV page
+                    const int32_t ra = kv_row_tma(a.pg, r0 + 128 * i);
+                    const int32_t rb = kv_row_tma(a.pg, r0 + 128 * i + 64);
+                    for (int hf = 0; hf < 2; ++hf) {
+                        uint8_t* dst = smem + kOffK + st * kTile + hf * kHalfT;
+                        tma_load_3d(dst, &tk, &bars.k_full[st], hf * 64, j, ra);
+                        tma_load_3d(dst + kHalfT / 2, &tk, &bars.k_full[st], hf * 64, j, rb);
+                    }
                 }
             }
             if (abort_flag) {
@@ -422,7 +428,8 @@ int tok_range(const Derived& d)
 }
 
 cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
-                                 const void* k, const float* fingerprints, const int32_t* unit_start,
+                                 const void* k, const KvPaging& pg, const float* fingerprints,
+                                 const int32_t* unit_start,
                                  const int32_t* n_units, int32_t* sel, int32_t* sel_count,
                                  float* sel_scores, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st)
 {
@@ -446,6 +453,7 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
     a.scores = sel_scores ? sel_scores : reinterpret_cast<float*>(ws + lay.scores);
     a.status = reinterpret_cast<int32_t*>(ws + kStatusOffset);
     a.timeout_ns = timeout_ns;
+    a.pg = pg;
     const int max_units = a.sc_end - a.sc_begin;
     if (max_units <= 0) return cudaSuccess;
 
@@ -454,7 +462,7 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
     const uint64_t fdims[4] = {kHeadDim, static_cast<uint64_t>(d.M) * d.g, static_cast<uint64_t>(d.Hkv), 3};
     const uint32_t fbox[4] = {64, 128, 1, 1};
     if (!scale_host::make_dense_bf16_map(&tf, parts, 4, fdims, fbox) ||
-        !scale_host::make_token_major_map(&tk, k, kHeadDim, d.Hkv, d.N, 64, 128))
+        !scale_host::make_token_major_map(&tk, k, kHeadDim, d.Hkv, pg.page_table ? pg.pool_rows : d.N, 64, 64))
         return cudaErrorInvalidValue;
 
     k_tok_split<<<static_cast<unsigned>(max_units) * d.Hq, 128, 0, st>>>(a, fingerprints, parts, static_cast<int>(d.M));

@@ -60,6 +60,20 @@ class ScaleParams(ctypes.Structure):
     ]
 
 
+class ScaleKvPages(ctypes.Structure):
+    """scale_kv_pages_t: a paged K/V cache (device pointers)."""
+
+    _fields_ = [("k_pages", ctypes.c_void_p), ("v_pages", ctypes.c_void_p),
+                ("page_table", ctypes.c_void_p), ("page_size", ctypes.c_int32),
+                ("num_pages", ctypes.c_int64)]
+
+
+def kv_pages(k_pages, v_pages, page_table, page_size: int) -> ScaleKvPages:
+    """Descriptor of torch tensors k_pages / v_pages [num_pages][page_size][H_kv][128]
+    and page_table (int32) on the device."""
+    return ScaleKvPages(_ptr(k_pages), _ptr(v_pages), _ptr(page_table), page_size, k_pages.shape[0])
+
+
 def params(*, num_q_heads, num_kv_heads, head_dim=128, sub_chunk, n_tokens, max_cluster_subchunks,
            outer_chunk=0, theta=-1.0, block_size, top_k, n_sink, n_local, select_scale=1.0,
            attn_scale=0.0) -> ScaleParams:
@@ -101,6 +115,7 @@ def load() -> ctypes.CDLL:
         lib = ctypes.CDLL(LIB_PATH)
         P, i32, i64, sz, u64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t, ctypes.c_uint64
         pp = ctypes.POINTER(ScaleParams)
+        kp = ctypes.POINTER(ScaleKvPages)
         sig = {
             "scale_workspace_size": [pp, i32, ctypes.POINTER(sz)],
             "scale_workspace_init": [P, sz, P],
@@ -108,6 +123,9 @@ def load() -> ctypes.CDLL:
             "scale_build_reps_noalloc": [pp, P, P, P, P, P, P, P],
             "scale_select": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, sz, P],
             "scale_select_tokens": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, sz, P],
+            "scale_build_reps_paged": [pp, P, kp, P, P, P, P, P, sz, P],
+            "scale_select_tokens_paged": [pp, i32, i64, i64, kp, P, P, P, P, P, P, P, sz, P],
+            "scale_sparse_prefill_paged": [pp, i32, i64, i64, P, kp, P, P, P, P, P, P, sz, P],
             "scale_sparse_prefill": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, P, sz, P],
             "scale_get_device_status": [P, P, ctypes.POINTER(i32)],
             "scale_retrieval_calls": [pp, i32, P, i32, ctypes.POINTER(i64), ctypes.POINTER(i64)],
@@ -220,6 +238,42 @@ def scale_sparse_prefill(p, mode, tok_begin, tok_end, q, k, v, unit_start, n_uni
         ctypes.byref(p), mode, tok_begin, tok_end, _ptr(q), _ptr(k), _ptr(v), _ptr(unit_start),
         _ptr(n_units), _ptr(sel_blocks), _ptr(sel_count), _ptr(out), _ptr(ws), _nbytes(ws),
         _stream(stream)))
+
+
+def scale_build_reps_paged(p, q, kv: ScaleKvPages, reps, fingerprints, unit_start, n_units, ws,
+                           stream=None) -> None:
+    _check("scale_build_reps_paged", load().scale_build_reps_paged(
+        ctypes.byref(p), _ptr(q), ctypes.byref(kv), _ptr(reps), _ptr(fingerprints), _ptr(unit_start),
+        _ptr(n_units), _ptr(ws), _nbytes(ws), _stream(stream)))
+
+
+def scale_select_tokens_paged(p, mode, tok_begin, tok_end, kv: ScaleKvPages, fingerprints, unit_start,
+                              n_units, sel_tokens, sel_count, sel_scores, ws, stream=None) -> None:
+    _check("scale_select_tokens_paged", load().scale_select_tokens_paged(
+        ctypes.byref(p), mode, tok_begin, tok_end, ctypes.byref(kv), _ptr(fingerprints), _ptr(unit_start),
+        _ptr(n_units), _ptr(sel_tokens), _ptr(sel_count), _ptr(sel_scores), _ptr(ws), _nbytes(ws),
+        _stream(stream)))
+
+
+def scale_sparse_prefill_paged(p, mode, tok_begin, tok_end, q, kv: ScaleKvPages, unit_start, n_units,
+                               sel_blocks, sel_count, out, ws, stream=None) -> None:
+    _check("scale_sparse_prefill_paged", load().scale_sparse_prefill_paged(
+        ctypes.byref(p), mode, tok_begin, tok_end, _ptr(q), ctypes.byref(kv), _ptr(unit_start),
+        _ptr(n_units), _ptr(sel_blocks), _ptr(sel_count), _ptr(out), _ptr(ws), _nbytes(ws),
+        _stream(stream)))
+
+
+def run_path_paged(p: ScaleParams, mode: int, q, kv: ScaleKvPages, buf: "Buffers", stream=None) -> None:
+    """Steps (a)-(d) with K and V in a paged cache."""
+    scale_build_reps_paged(p, q, kv, buf.reps, buf.fingerprints, buf.unit_start, buf.n_units, buf.ws, stream)
+    if p.block_size == 1:
+        scale_select_tokens_paged(p, mode, 0, p.n_tokens, kv, buf.fingerprints, buf.unit_start, buf.n_units,
+                                  buf.sel_blocks, buf.sel_count, buf.sel_scores, buf.ws, stream)
+    else:
+        scale_select(p, mode, 0, p.n_tokens, buf.reps, buf.fingerprints, buf.unit_start, buf.n_units,
+                     buf.sel_blocks, buf.sel_count, buf.sel_scores, buf.ws, stream)
+    scale_sparse_prefill_paged(p, mode, 0, p.n_tokens, q, kv, buf.unit_start, buf.n_units, buf.sel_blocks,
+                               buf.sel_count, buf.out, buf.ws, stream)
 
 
 def scale_get_device_status(ws, stream=None) -> int:

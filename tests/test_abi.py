@@ -162,3 +162,45 @@ def test_token_workspace_has_no_logits_plane():
     big = M * N * 4 + 2 * M * w.num_kv_heads * slots * 128 * 2
     assert big <= n < big * 1.1
     assert n < M * w.num_q_heads * N * 4  # the logits plane alone would be larger
+
+
+def test_kv_pages_struct_layout_matches_header():
+    src = r"""
+#include <stddef.h>
+#include <stdio.h>
+#include "scale.h"
+#define F(x) printf(#x " %zu\n", offsetof(scale_kv_pages_t, x));
+int main(void) {
+  printf("size %zu\n", sizeof(scale_kv_pages_t));
+  F(k_pages) F(v_pages) F(page_table) F(page_size) F(num_pages)
+  return 0;
+}
+"""
+    with tempfile.TemporaryDirectory() as d:
+        c = os.path.join(d, "t.c")
+        exe = os.path.join(d, "t")
+        with open(c, "w") as f:
+            f.write(src)
+        subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), c, "-o", exe], check=True)
+        out = subprocess.run([exe], capture_output=True, text=True, check=True).stdout
+    got = dict(line.split() for line in out.strip().splitlines())
+    assert int(got.pop("size")) == ctypes.sizeof(S.ScaleKvPages)
+    for name, off in got.items():
+        assert getattr(S.ScaleKvPages, name).offset == int(off), name
+
+
+@pytest.mark.parametrize("page_size,over,rc", [
+    (100, {}, S.SCALE_ERR_UNSUPPORTED),                 # pages of 64-row boxes only
+    (64, dict(n_sink=100), S.SCALE_ERR_UNSUPPORTED),    # sinks must end on a 64-row boundary
+    (64, dict(block_size=96), S.SCALE_ERR_UNSUPPORTED),
+    (0, {}, S.SCALE_ERR_INVALID_ARG),
+    (64, {}, S.SCALE_ERR_INVALID_ARG),                  # valid sizes, null pointers
+])
+def test_paged_entry_points_validate_before_launch(lib, page_size, over, rc):
+    p = _p(**over)
+    kv = S.ScaleKvPages(None, None, None, page_size, 16)
+    assert lib.scale_sparse_prefill_paged(ctypes.byref(p), 0, 0, p.n_tokens, None, ctypes.byref(kv), None,
+                                          None, None, None, None, None, 0, None) == rc
+    assert lib.scale_build_reps_paged(ctypes.byref(p), None, ctypes.byref(kv), None, None, None, None,
+                                      None, 0, None) == rc
+

@@ -522,3 +522,68 @@ def test_1m_context_full_size():
         n, mx, mean, near = _full_size_check(w, q, k, v, mode, n_random=40)
         print(f"1M mode={mode}: {n} rows, max {mx:.3e} mean {mean:.3e}, {near} near-tie units")
         assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+# --------------------------------------------------------------------------- paged KV cache
+
+
+def _paged(x, page_size, rng, extra=3):
+    """x [N][H][128] on the device -> (pool [n_pages + extra][P][H][128], page table):
+    pages in shuffled order, unused pages and the tail of the last page filled
+    with large values that a wrong read would expose."""
+    N, H, D = x.shape
+    n_pages = -(-N // page_size)
+    pool = torch.full((n_pages + extra, page_size, H, D), 1000.0, dtype=x.dtype, device=x.device)
+    perm = torch.from_numpy(rng.permutation(n_pages + extra)[:n_pages].astype(np.int32)).to(x.device)
+    for i in range(n_pages):
+        rows = x[i * page_size:(i + 1) * page_size]
+        pool[int(perm[i]), : rows.shape[0]] = rows
+    return pool, perm
+
+
+PAGED_CASES = [("gqa4-4k", {}, 64), ("gqa4-4k", dict(n_tokens=3000), 128),
+               ("llama8b-32k", {}, 256), ("llama8b-32k", dict(block_size=1, top_k=1024), 128)]
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+@pytest.mark.parametrize("name,over,page", PAGED_CASES)
+def test_paged_kv_equals_contiguous(name, over, page, mode):
+    """The *_paged entry points on a shuffled page pool give the contiguous
+    path's results bit for bit (same keys and values, same arithmetic)."""
+    w, q, k, v, dev = inputs(name, **over)
+    p, ref = gpu_path(w, mode, dev)
+    rng = np.random.default_rng(11)
+    kp, table = _paged(dev[1], page, rng)
+    vp, _ = _paged(dev[2], page, np.random.default_rng(11))
+    kv = S.kv_pages(kp, vp, table, page)
+    buf = S.allocate(p, mode)
+    S.run_path_paged(p, mode, dev[0], kv, buf)
+    torch.cuda.synchronize()
+    assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
+    if w.block_size > 1:
+        assert torch.equal(buf.reps, ref.reps)
+    assert torch.equal(buf.fingerprints, ref.fingerprints)
+    n = unit_count(ref, mode, w)
+    assert torch.equal(buf.sel_count[:n], ref.sel_count[:n])
+    assert torch.equal(buf.sel_blocks[:n], ref.sel_blocks[:n])
+    assert torch.equal(buf.out, ref.out)
+
+
+def test_paged_kv_entry_outside_pool_reads_zeros():
+    """A page-table entry outside the pool is not dereferenced; its tokens act
+    as zero keys and values (checked against the contiguous path with those
+    rows zeroed)."""
+    w, q, k, v, dev = inputs("gqa4-4k")
+    page = 64
+    kz, vz = dev[1].clone(), dev[2].clone()
+    kz[3 * page:4 * page] = 0
+    vz[3 * page:4 * page] = 0
+    p, ref = gpu_path(w, PER_CLUSTER, [dev[0], kz, vz])
+    kp, table = _paged(dev[1], page, np.random.default_rng(5))
+    vp, _ = _paged(dev[2], page, np.random.default_rng(5))
+    table[3] = kp.shape[0] + 7
+    buf = S.allocate(p, PER_CLUSTER)
+    S.run_path_paged(p, PER_CLUSTER, dev[0], S.kv_pages(kp, vp, table, page), buf)
+    torch.cuda.synchronize()
+    assert torch.equal(buf.reps, ref.reps)
+    assert torch.equal(buf.out, ref.out)
