@@ -51,6 +51,8 @@ def parse_args():
                     help="target CPU time of the oracle sample")
     ap.add_argument("--paged", type=int, default=0, metavar="P",
                     help="keep K and V in a paged cache of P-token pages (shuffled page order)")
+    ap.add_argument("--decode", action="store_true",
+                    help="decode steps with the selection cache at the end of the context (one JSON line)")
     ap.add_argument("--sweep", action="store_true",
                     help="clustering-threshold sweep (theta x L_max) on planted-topic data: cluster sizes, "
                          "overlap ratio rho, boundary recall and step time (one JSON line)")
@@ -587,6 +589,67 @@ def run_sweep(args):
     return 0
 
 
+DECODE_WORKLOAD = "llama8b-1m-tok"
+
+
+def run_decode(args):
+    """Decode steps at the end of the context: every step retrieving (no
+    cache) against the selection cache reusing a retrieval for up to 16 steps.
+    Queries are a random walk from the last prompt query (consecutive decode
+    queries are close); K and V are the workload's. Attention-only TPOT."""
+    import torch
+
+    import paper_2609_31568_gb300 as pkg
+    from paper_2609_31568_gb300 import scale as S
+    from synth import bf16_bits_to_f32, f64_to_bf16_bits
+
+    pkg.build()
+    S.load()
+    w = workload(args.workload if args.workload != DEFAULT_WORKLOAD else DECODE_WORKLOAD)
+    n_steps = 64
+    q, k, v = generate_layer(w)
+    rng = np.random.default_rng(3)
+    x = bf16_bits_to_f32(q[w.n_tokens - n_steps]).astype(np.float64)
+    walk = []
+    for _ in range(n_steps):
+        walk.append(f64_to_bf16_bits(x))
+        x = x + 0.07 * np.linalg.norm(x) / np.sqrt(x.size) * rng.standard_normal(x.shape)
+    qd = torch.from_numpy(np.stack(walk)).view(torch.bfloat16).cuda()
+    kd, vd = (torch.from_numpy(t).view(torch.bfloat16).cuda() for t in (k, v))
+    del q
+    positions = list(range(w.n_tokens - n_steps, w.n_tokens))
+    stream = torch.cuda.current_stream()
+    res = {}
+    for label, theta, s_max in (("retrieve_every_step", 2.0, 1), ("selection_cache", -1.0, 16)):
+        p = S.params_for(w, theta=theta, max_cluster_subchunks=s_max)
+        cache = torch.empty(S.scale_decode_cache_size(p), dtype=torch.uint8, device="cuda")
+        ws = torch.empty(S.scale_decode_workspace_size(p), dtype=torch.uint8, device="cuda")
+        out = torch.empty((w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+        for _ in range(max(1, args.warmup)):
+            S.scale_decode_cache_init(cache)
+            for i, t in enumerate(positions[:8]):
+                S.scale_decode_step(p, t, qd[i], kd, vd, cache, out, ws, stream)
+        torch.cuda.synchronize()
+        S.scale_decode_cache_init(cache)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(n_steps + 1)]
+        ev[0].record(stream)
+        for i, t in enumerate(positions):
+            S.scale_decode_step(p, t, qd[i], kd, vd, cache, out, ws, stream)
+            ev[i + 1].record(stream)
+        torch.cuda.synchronize()
+        ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(n_steps)]
+        res[label] = {"tpot_ms": statistics.mean(ms), "retrieving_step_ms": ms[0],
+                      "reusing_step_ms": statistics.median(ms[1:]) if s_max > 1 else None,
+                      "retrievals": -(-n_steps // s_max)}
+    line = {"metric": "decode TPOT (attention only) with the selection cache", "workload": w.name,
+            "context": w.n_tokens, "top_k_tokens": w.top_k, "steps": n_steps,
+            "value": 1000.0 / res["selection_cache"]["tpot_ms"], "unit": "tokens/s",
+            "speedup_from_cache": res["retrieve_every_step"]["tpot_ms"] / res["selection_cache"]["tpot_ms"],
+            "data": "synthetic (random-walk decode queries)", **res}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_stack(args):
     """Multi-layer workload: attention-only TTFT of a chunked prefill over all layers.
 
@@ -715,6 +778,8 @@ def main():
         return run_reference(args)
     if args.sweep:
         return run_sweep(args)
+    if args.decode:
+        return run_decode(args)
     if workload(args.workload).layers > 1:
         return run_stack(args)
     return run_scale(args)

@@ -247,6 +247,34 @@ int scale_sparse_prefill_paged(const scale_params_t *p, int32_t mode, int64_t to
                                const int32_t *sel_blocks, const int32_t *sel_count, void *out,
                                void *ws, size_t ws_bytes, scale_stream_t stream);
 
+/* One decode step with a selection cache. The paper's method targets prefill
+ * and leaves decode to its engine, whose selection cache reuses a token
+ * selection across consecutive, highly similar decode queries (Sec. VII).
+ * This step applies the paper's rules with one query token (Def. 1, C = 1):
+ *  - the query q_t of position t (its K and V rows already at row t) is the
+ *    unit's fingerprint; its candidates are the tokens n_sink <= c < W_t,
+ *    W_t = max(0, t - n_local);
+ *  - reuse: with an anchor in `cache`, the step reuses the anchor's selection
+ *    when cos(q_t, anchor) >= theta (all heads together, as Eq. 8; a zero norm
+ *    gives cosine 0) and fewer than max_cluster_subchunks steps have shared
+ *    it; otherwise it retrieves (Eq. 9 at block size 1: per-head softmax over
+ *    the candidates, head soft-vote, top_k tokens, ties to the lower index)
+ *    and q_t becomes the anchor;
+ *  - out_t[h] = Eq. 10 for the single row t over sinks U selection U [W_t, t].
+ * Parameters: n_tokens = rows of k and v (t < n_tokens), block_size must be
+ * 1, H_q / H_kv at most 8, H_q at most 96; sub_chunk and outer_chunk are not
+ * used. The reuse decision is made on the device: a step never synchronises.
+ *   q_t, out_t  bf16 [H_q][128];  k, v  bf16 [n_tokens][H_kv][128]
+ *   cache       scale_decode_cache_size() bytes, zeroed by
+ *               scale_decode_cache_init() before the first step of a sequence
+ *   ws          scale_decode_workspace_size() bytes (grows with n_tokens) */
+int scale_decode_cache_size(const scale_params_t *p, size_t *bytes);
+int scale_decode_cache_init(void *cache, size_t cache_bytes, scale_stream_t stream);
+int scale_decode_workspace_size(const scale_params_t *p, size_t *bytes);
+int scale_decode_step(const scale_params_t *p, int64_t t, const void *q_t, const void *k, const void *v,
+                      void *cache, size_t cache_bytes, void *out_t, void *ws, size_t ws_bytes,
+                      scale_stream_t stream);
+
 /* Synchronous: waits for `stream`, then reads the device status word of `ws`
  * into *status (SCALE_OK, SCALE_ERR_TIMEOUT or SCALE_ERR_DEVICE). The word is
  * sticky until scale_workspace_init(). */

@@ -224,3 +224,68 @@ def overlap_ratio(anchor_blocks, member_blocks) -> float:
         others |= {int(b) for b in m}
     return len(anchor & others) / len(anchor)
 
+
+def _bf16_f64(x: np.ndarray) -> np.ndarray:
+    x = np.ascontiguousarray(x, np.uint16)
+    return (x.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+
+
+def decode_select(q_t: np.ndarray, k: np.ndarray, t: int, *, n_sink: int, n_local: int, top_k: int,
+                  select_scale: float = 1.0):
+    """Eq. 9 for one query token (a unit of C = 1 token, Def. 1) at position t,
+    token level: candidates n_sink <= c < W_t = max(0, t - n_local); per-head
+    softmax of select_scale * q^(h) . k_c^(h / g) over them, summed over the
+    heads; the top_k tokens by (score desc, index asc), returned ascending,
+    with the relative gap between the k-th and (k+1)-th scores (inf if none).
+      q_t [H_q][d] bf16 bits, k [N][H_kv][d] bf16 bits."""
+    Hq = q_t.shape[0]
+    Hkv = k.shape[1]
+    g = Hq // Hkv
+    W = max(0, t - n_local)
+    cand = np.arange(n_sink, W, dtype=np.int64)
+    if cand.size == 0:
+        return np.zeros(0, np.int64), np.inf
+    q = _bf16_f64(q_t)
+    kc = _bf16_f64(k[cand])  # [n, H_kv, d]
+    score = np.zeros(cand.size)
+    for h in range(Hq):
+        z = select_scale * (kc[:, h // g, :] @ q[h])
+        e = np.exp(z - z.max())
+        score += e / e.sum()
+    order = np.lexsort((cand, -score))
+    take = min(top_k, cand.size)
+    gap = np.inf
+    if cand.size > top_k > 0:
+        s_k, s_k1 = score[order[top_k - 1]], score[order[top_k]]
+        gap = (s_k - s_k1) / s_k
+    return np.sort(cand[order[:take]]), gap
+
+
+def decode_reuse(queries: np.ndarray, theta: float, max_shared: int):
+    """The selection cache across decode steps (Eq. 8 with Algorithm 1's cap,
+    applied in time): step 0 retrieves; step i reuses the anchor's selection
+    when cos(q_i, anchor) >= theta (all heads together; a zero norm gives 0)
+    and fewer than max_shared steps have shared it, else it retrieves and
+    becomes the anchor. Returns (retrieve flags, anchor index of every step,
+    |cos - theta| of the closest decision).
+      queries [T][H_q][d] bf16 bits."""
+    qs = [_bf16_f64(q).ravel() for q in queries]
+    retrieve, anchor_of, margin = [], [], np.inf
+    anchor, shared = None, 0
+    for i, q in enumerate(qs):
+        if anchor is None:
+            reuse = False
+        else:
+            na, nq = np.linalg.norm(qs[anchor]), np.linalg.norm(q)
+            c = float(qs[anchor] @ q / (na * nq)) if na > 0 and nq > 0 else 0.0
+            if shared < max_shared:
+                margin = min(margin, abs(c - theta))
+            reuse = shared < max_shared and c >= theta
+        if reuse:
+            shared += 1
+        else:
+            anchor, shared = i, 1
+        retrieve.append(not reuse)
+        anchor_of.append(anchor)
+    return np.array(retrieve), np.array(anchor_of), margin
+

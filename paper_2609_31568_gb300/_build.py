@@ -18,7 +18,7 @@ LIB = os.path.join(HERE, "libscale.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
               "-Xptxas", "-v", "--use_fast_math", "-DNDEBUG"]
-SOURCES = ["api.cu", "reps.cu", "select.cu", "select_tok.cu", "attn.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "reps.cu", "select.cu", "select_tok.cu", "attn.cu", "noalloc.cu", "decode.cu"]
 HEADERS = ["scale_internal.h", "ptx_sm103.cuh", "tma_host.h"]
 
 

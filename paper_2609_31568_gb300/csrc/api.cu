@@ -453,6 +453,51 @@ int scale_prefill_host(const scale_params_t* p, int32_t mode, const void* q_host
     return st;
 }
 
+int scale_decode_cache_size(const scale_params_t* p, size_t* bytes)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (!bytes) return SCALE_ERR_INVALID_ARG;
+    *bytes = align_up(decode_cache_bytes(d), kAlign);
+    return SCALE_OK;
+}
+
+int scale_decode_cache_init(void* cache, size_t cache_bytes, scale_stream_t stream)
+{
+    if (!device_ptr(cache, 256) || cache_bytes < 256) return SCALE_ERR_INVALID_ARG;
+    return cuda_status(cudaMemsetAsync(cache, 0, cache_bytes, stream));
+}
+
+int scale_decode_workspace_size(const scale_params_t* p, size_t* bytes)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (!bytes) return SCALE_ERR_INVALID_ARG;
+    *bytes = decode_ws_bytes(d, decode_splits());
+    return SCALE_OK;
+}
+
+int scale_decode_step(const scale_params_t* p, int64_t t, const void* q_t, const void* k, const void* v,
+                      void* cache, size_t cache_bytes, void* out_t, void* ws, size_t ws_bytes,
+                      scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if (d.B != 1) return SCALE_ERR_INVALID_ARG;
+    if (d.g > 8 || d.Hq > 96) return SCALE_ERR_UNSUPPORTED;
+    if (t < 0 || t >= d.N) return SCALE_ERR_INVALID_ARG;
+    if (!device_ptr(q_t, 16) || !device_ptr(k, 16) || !device_ptr(v, 16) || !device_ptr(out_t, 16) ||
+        !device_ptr(cache, 256) || !device_ptr(ws, 256))
+        return SCALE_ERR_INVALID_ARG;
+    if (cache_bytes < decode_cache_bytes(d) || ws_bytes < decode_ws_bytes(d, decode_splits()))
+        return SCALE_ERR_WORKSPACE;
+    return cuda_status(launch_decode_step(d, t, q_t, k, v, static_cast<uint8_t*>(cache), out_t,
+                                          static_cast<uint8_t*>(ws), stream));
+}
+
 int scale_set_wait_timeout_ns(uint64_t ns)
 {
     if (ns == 0) return SCALE_ERR_INVALID_ARG;

@@ -163,7 +163,7 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
                                   uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 cudaError_t launch_wait_selftest(uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_end, const float* scores,
-                        int32_t* sel, int32_t* sel_count, cudaStream_t st);
+                        int32_t* sel, int32_t* sel_count, cudaStream_t st, const int32_t* gate = nullptr);
 cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
                                  const void* k, const KvPaging& pg, const float* fingerprints,
                                  const int32_t* unit_start,
@@ -171,6 +171,12 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
                                  float* sel_scores, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 // Tokens per CTA of the token-level scoring kernels.
 int tok_range(const Derived& d);
+// Decode step (decode.cu).
+size_t decode_cache_bytes(const Derived& d);
+size_t decode_ws_bytes(const Derived& d, int splits);
+int decode_splits();
+cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const void* k, const void* v,
+                               uint8_t* cache, void* out, uint8_t* ws, cudaStream_t st);
 
 // Packed distant rows per (unit, KV head) at block size 1: n_sink + k rounded
 // up to a multiple of 128.

@@ -28,6 +28,7 @@ struct SelArgs {
     int64_t nb;
     int B, k, n_sink, n_local;
     float sigma;
+    const int32_t* gate;  // nullable: the top-k runs only when *gate != 0
 };
 
 __device__ __forceinline__ void cand_range(const SelArgs& a, int64_t s, int64_t* lo, int64_t* hi)
@@ -190,6 +191,7 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
     __shared__ int whist[kTopkThreads / 32][256];  // per-warp histograms
     __shared__ uint32_t s_prefix;
     __shared__ int s_need;
+    if (a.gate && !*a.gate) return;
     const int u_first = unit_lower_bound(a.ut, a.sc_begin);
     const int u_end = unit_lower_bound(a.ut, a.sc_end);
     const int u = u_first + blockIdx.x;
@@ -357,7 +359,7 @@ cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t
     float* stats = reinterpret_cast<float*>(ws + lay.stats);
     float* scores = sel_scores ? sel_scores : reinterpret_cast<float*>(ws + lay.scores);
 
-    SelArgs a;
+    SelArgs a{};
     a.ut = Units{unit_start, n_units, mode == SCALE_MODE_PER_SUBCHUNK, d.N, d.L, static_cast<int>(d.M)};
     a.sc_begin = static_cast<int>(tok_begin / d.L);
     a.sc_end = static_cast<int>((tok_end + d.L - 1) / d.L);
@@ -391,9 +393,10 @@ cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t
 }
 
 cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_end, const float* scores,
-                        int32_t* sel, int32_t* sel_count, cudaStream_t st)
+                        int32_t* sel, int32_t* sel_count, cudaStream_t st, const int32_t* gate)
 {
     SelArgs a{};
+    a.gate = gate;
     a.ut = ut;
     a.sc_begin = sc_begin;
     a.sc_end = sc_end;

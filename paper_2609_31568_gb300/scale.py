@@ -126,6 +126,10 @@ def load() -> ctypes.CDLL:
             "scale_build_reps_paged": [pp, P, kp, P, P, P, P, P, sz, P],
             "scale_select_tokens_paged": [pp, i32, i64, i64, kp, P, P, P, P, P, P, P, sz, P],
             "scale_sparse_prefill_paged": [pp, i32, i64, i64, P, kp, P, P, P, P, P, P, sz, P],
+            "scale_decode_cache_size": [pp, ctypes.POINTER(sz)],
+            "scale_decode_cache_init": [P, sz, P],
+            "scale_decode_workspace_size": [pp, ctypes.POINTER(sz)],
+            "scale_decode_step": [pp, i64, P, P, P, P, sz, P, P, sz, P],
             "scale_sparse_prefill": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, P, sz, P],
             "scale_get_device_status": [P, P, ctypes.POINTER(i32)],
             "scale_retrieval_calls": [pp, i32, P, i32, ctypes.POINTER(i64), ctypes.POINTER(i64)],
@@ -274,6 +278,47 @@ def run_path_paged(p: ScaleParams, mode: int, q, kv: ScaleKvPages, buf: "Buffers
                      buf.sel_blocks, buf.sel_count, buf.sel_scores, buf.ws, stream)
     scale_sparse_prefill_paged(p, mode, 0, p.n_tokens, q, kv, buf.unit_start, buf.n_units, buf.sel_blocks,
                                buf.sel_count, buf.out, buf.ws, stream)
+
+
+def scale_decode_cache_size(p) -> int:
+    n = ctypes.c_size_t()
+    _check("scale_decode_cache_size", load().scale_decode_cache_size(ctypes.byref(p), ctypes.byref(n)))
+    return n.value
+
+
+def scale_decode_cache_init(cache, stream=None) -> None:
+    _check("scale_decode_cache_init", load().scale_decode_cache_init(_ptr(cache), _nbytes(cache), _stream(stream)))
+
+
+def scale_decode_workspace_size(p) -> int:
+    n = ctypes.c_size_t()
+    _check("scale_decode_workspace_size", load().scale_decode_workspace_size(ctypes.byref(p), ctypes.byref(n)))
+    return n.value
+
+
+def scale_decode_step(p, t: int, q_t, k, v, cache, out_t, ws, stream=None) -> None:
+    _check("scale_decode_step", load().scale_decode_step(
+        ctypes.byref(p), t, _ptr(q_t), _ptr(k), _ptr(v), _ptr(cache), _nbytes(cache), _ptr(out_t),
+        _ptr(ws), _nbytes(ws), _stream(stream)))
+
+
+def decode_cache_state(cache) -> dict:
+    """Host view of a decode cache's header: whether the last step retrieved,
+    the anchor position, steps sharing the anchor, and its selection size."""
+    import torch
+
+    st = cache[:64].view(torch.int32).cpu().tolist()
+    return {"valid": st[0], "steps": st[1], "retrieved": st[2], "anchor": st[4]}
+
+
+def decode_cache_selection(cache, p) -> tuple:
+    """The selection held by a decode cache (ascending tokens) and its size."""
+    import torch
+
+    off = 256 + p.num_q_heads * 128 * 4
+    k = max(p.top_k, 1)
+    raw = cache[off: off + (k + 1) * 4].view(torch.int32).cpu().numpy()
+    return raw[:k].copy(), int(raw[k])
 
 
 def scale_get_device_status(ws, stream=None) -> int:

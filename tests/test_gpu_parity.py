@@ -587,3 +587,86 @@ def test_paged_kv_entry_outside_pool_reads_zeros():
     torch.cuda.synchronize()
     assert torch.equal(buf.reps, ref.reps)
     assert torch.equal(buf.out, ref.out)
+
+
+# --------------------------------------------------------------------------- decode with a selection cache
+
+
+def _decode_queries(q, steps, seed=3):
+    """Decode queries as consecutive generated tokens behave: a random walk from
+    the query row at the first step (bf16), each step moving by about 7 % of
+    its norm, so consecutive queries are close and drift apart with distance."""
+    from synth import bf16_bits_to_f32, f64_to_bf16_bits
+
+    rng = np.random.default_rng(seed)
+    x = bf16_bits_to_f32(q[steps[0]]).astype(np.float64)
+    scale = 0.07 * np.linalg.norm(x) / np.sqrt(x.size)
+    out = []
+    for _ in steps:
+        out.append(f64_to_bf16_bits(x))
+        x = x + scale * rng.standard_normal(x.shape)
+    return np.stack(out)
+
+
+def _decode_theta(qd, s_max):
+    """A reuse threshold under which the cosine, not only the cap, decides some
+    steps, with a mix of decisions and every decision far (> 1e-4) from it."""
+    cap_only, _, _ = oracle.decode_reuse(qd, -1.0, s_max)
+    best = None
+    for theta in np.linspace(0.90, 0.999, 100):
+        r, _, margin = oracle.decode_reuse(qd, float(theta), s_max)
+        if (not np.array_equal(r, cap_only) and 2 < (~r).sum() < len(r) - 4 and margin > 1e-4
+                and (best is None or margin > best[1])):
+            best = (float(theta), margin)
+    assert best is not None
+    return best[0]
+
+
+@pytest.mark.parametrize("theta", [-1.0, None])
+def test_decode_steps_with_selection_cache(theta):
+    """scale_decode_step over 40 consecutive positions: reuse decisions, the
+    selection of every retrieving step and every output row against the oracle."""
+    w, q, k, v, dev = inputs("llama8b-32k", n_tokens=4096, block_size=1, top_k=256, n_local=512)
+    steps = np.arange(3000, 3040)
+    s_max = 8
+    qd = _decode_queries(q, steps)
+    if theta is None:
+        theta = _decode_theta(qd, s_max)
+    p = S.params_for(w, theta=theta, max_cluster_subchunks=s_max)
+    cache = torch.empty(S.scale_decode_cache_size(p), dtype=torch.uint8, device="cuda")
+    S.scale_decode_cache_init(cache)
+    ws = torch.empty(S.scale_decode_workspace_size(p), dtype=torch.uint8, device="cuda")
+    qd_dev = torch.from_numpy(qd).view(torch.bfloat16).cuda()
+    want_r, anchor_of, margin = oracle.decode_reuse(qd, theta, s_max)
+    assert margin > 1e-5
+    sel_full = np.full((w.n_tokens, w.top_k), -1, np.int32)
+    cnt_full = np.zeros(w.n_tokens, np.int32)
+    outs, near = [], 0
+    for i, t in enumerate(steps):
+        out = torch.empty((w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
+        S.scale_decode_step(p, int(t), qd_dev[i], dev[1], dev[2], cache, out, ws)
+        torch.cuda.synchronize()
+        st = S.decode_cache_state(cache)
+        assert bool(st["retrieved"]) == bool(want_r[i]), f"step {t}"
+        assert st["anchor"] == steps[anchor_of[i]]
+        sel, cnt = S.decode_cache_selection(cache, p)
+        if want_r[i]:
+            ref, gap = oracle.decode_select(qd[i], k, int(t), n_sink=w.n_sink, n_local=w.n_local,
+                                            top_k=w.top_k)
+            assert cnt == len(ref)
+            if sel[:cnt].tolist() != ref.tolist():
+                assert gap < NEAR_TIE_GAP, f"step {t}: selection differs with gap {gap:.3e}"
+                near += 1
+        sel_full[t, :cnt] = sel[:cnt]
+        cnt_full[t] = cnt
+        outs.append(to_f64_bf16(out))
+    q_rows = q.copy()
+    q_rows[steps] = qd
+    ref_attn = oracle.attention_rows(q=q_rows, k=k, v=v, sub_chunk=1, block_size=1, top_k=w.top_k,
+                                     n_sink=w.n_sink, n_local=w.n_local,
+                                     attn_scale=1.0 / np.sqrt(w.head_dim), per_subchunk=True,
+                                     unit_start=None, sel=sel_full, sel_count=cnt_full, rows=steps)
+    mx, mean = attn_errors(np.stack(outs), ref_attn)
+    print(f"theta={theta:.4f}: {int(want_r.sum())} retrievals in {len(steps)} steps, {near} near-ties, "
+          f"attention max {mx:.3e} mean {mean:.3e}")
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
