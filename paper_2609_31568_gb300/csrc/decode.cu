@@ -51,10 +51,10 @@ struct DecArgs {
     float* z;           // [H_q][cap]
     float2* stats;      // [H_q] (max, 1 / sum)
     float* scores;      // [cap]
-    int32_t* list;      // distant + window keys of this step
-    int32_t* list_n;
     float* part;        // [H_q][splits][130]: max, sum, o[128]
     int splits;
+    float2* zpart;      // [chunks][H_q] (max, sum) of each candidate chunk
+    int chunk;          // candidates per logits CTA
 };
 
 __host__ __device__ __forceinline__ int64_t window_start(const DecArgs& a, int64_t t)
@@ -117,59 +117,80 @@ __global__ void __launch_bounds__(256) k_dec_gate(DecArgs a, const __nv_bfloat16
         for (int i = threadIdx.x; i < D; i += blockDim.x) a.anchor[i] = __bfloat162float(q[i]);
 }
 
-// z[h][c] = sigma * q^(h) . k_c^(h / g) for the candidates c; one warp per key,
-// lane l holding dimensions [4 l, 4 l + 4) of every head.
-__global__ void __launch_bounds__(256) k_dec_logits(DecArgs a, const __nv_bfloat16* __restrict__ q,
-                                                    const uint2* __restrict__ k)
+// z[h][c] = sigma * q^(h) . k_c^(h / g) for the candidates c of this CTA's
+// chunk [lo + chunk * blockIdx.x, + chunk): one thread per key, streaming its
+// K row in 16-byte pieces (the query, in shared memory, is read as
+// broadcasts). The chunk's logits are staged in shared memory, written out as
+// whole rows, and summarised per head as (max, sum of exp(z - max)).
+__global__ void __launch_bounds__(128) k_dec_logits(DecArgs a, const __nv_bfloat16* __restrict__ q,
+                                                    const uint4* __restrict__ k)
 {
     if (!a.state[2]) return;
-    extern __shared__ float qs[];  // [H_q][128]
+    extern __shared__ float sm[];
+    float* qs = sm;                        // [H_q][128]
+    float* zs = sm + a.Hq * kHeadDim;      // [H_q][chunk]
     const int D = a.Hq * kHeadDim;
     for (int i = threadIdx.x; i < D; i += blockDim.x) qs[i] = __bfloat162float(q[i]);
     __syncthreads();
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int64_t lo = a.n_sink, hi = window_start(a, a.t);
-    for (int64_t c = lo + static_cast<int64_t>(blockIdx.x) * 8 + warp; c < hi; c += static_cast<int64_t>(gridDim.x) * 8) {
+    const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * a.chunk;
+    const int n = static_cast<int>((hi - c0 < a.chunk) ? hi - c0 : a.chunk);
+    const int i = threadIdx.x;
+    if (i < n) {
+        const int64_t c = c0 + i;
         for (int j = 0; j < a.Hkv; ++j) {
-            const uint2 kw = k[(c * a.Hkv + j) * 32 + lane];  // 4 bf16 of this lane
-            const float k0 = bf16_lo(kw.x), k1 = bf16_hi(kw.x), k2 = bf16_lo(kw.y), k3 = bf16_hi(kw.y);
+            const uint4* kr = k + (c * a.Hkv + j) * 16;  // 16 pieces of 8 bf16
+            uint4 kv[16];
+#pragma unroll
+            for (int p = 0; p < 16; ++p) kv[p] = kr[p];
             for (int hl = 0; hl < a.g; ++hl) {
-                const int h = j * a.g + hl;
-                const float* qh = qs + h * kHeadDim + 4 * lane;
-                float d = qh[0] * k0 + qh[1] * k1 + qh[2] * k2 + qh[3] * k3;
-                for (int o = 16; o > 0; o >>= 1) d += __shfl_xor_sync(0xFFFFFFFFu, d, o);
-                if (lane == 0) a.z[h * a.cap + c] = a.sigma * d;
+                const float4* qh = reinterpret_cast<const float4*>(qs + (j * a.g + hl) * kHeadDim);
+                float acc = 0.f;
+#pragma unroll
+                for (int p = 0; p < 16; ++p) {
+                    const float4 qa = qh[2 * p], qb = qh[2 * p + 1];
+                    acc += qa.x * bf16_lo(kv[p].x) + qa.y * bf16_hi(kv[p].x) + qa.z * bf16_lo(kv[p].y) +
+                           qa.w * bf16_hi(kv[p].y) + qb.x * bf16_lo(kv[p].z) + qb.y * bf16_hi(kv[p].z) +
+                           qb.z * bf16_lo(kv[p].w) + qb.w * bf16_hi(kv[p].w);
+                }
+                zs[(j * a.g + hl) * a.chunk + i] = a.sigma * acc;
             }
         }
     }
+    __syncthreads();
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int h = warp; h < a.Hq; h += blockDim.x / 32) {
+        const float* zh = zs + h * a.chunk;
+        float* dst = a.z + h * a.cap + c0;
+        float m = -INFINITY;
+        for (int ii = lane; ii < n; ii += 32) {
+            dst[ii] = zh[ii];
+            m = fmaxf(m, zh[ii]);
+        }
+        for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+        float sum = 0.f;
+        for (int ii = lane; ii < n; ii += 32) sum += expf(zh[ii] - m);
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+        if (lane == 0) a.zpart[static_cast<int64_t>(blockIdx.x) * a.Hq + h] = make_float2(m, sum);
+    }
 }
 
-// Per head: max of z over the candidates and 1 / sum of exp(z - max).
-__global__ void __launch_bounds__(256) k_dec_stats(DecArgs a)
+// Per head (one warp): the chunks' (max, sum) merged into max and 1 / sum.
+__global__ void __launch_bounds__(256) k_dec_stats(DecArgs a, int n_chunks)
 {
     if (!a.state[2]) return;
-    __shared__ float red[8];
-    const int h = blockIdx.x;
-    const int64_t lo = a.n_sink, hi = window_start(a, a.t);
-    const float* zh = a.z + h * a.cap;
+    const int h = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+    if (h >= a.Hq) return;
     float m = -INFINITY;
-    for (int64_t c = lo + threadIdx.x; c < hi; c += blockDim.x) m = fmaxf(m, zh[c]);
+    for (int b = lane; b < n_chunks; b += 32) m = fmaxf(m, a.zpart[static_cast<int64_t>(b) * a.Hq + h].x);
     for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
-    __syncthreads();
-    m = red[0];
-    for (int i = 1; i < 8; ++i) m = fmaxf(m, red[i]);
-    __syncthreads();
     float s = 0.f;
-    for (int64_t c = lo + threadIdx.x; c < hi; c += blockDim.x) s += expf(zh[c] - m);
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        float t = 0.f;
-        for (int i = 0; i < 8; ++i) t += red[i];
-        a.stats[h] = make_float2(m, t > 0.f ? 1.0f / t : 0.f);
+    for (int b = lane; b < n_chunks; b += 32) {
+        const float2 p = a.zpart[static_cast<int64_t>(b) * a.Hq + h];
+        if (p.x > -INFINITY) s += p.y * expf(p.x - m);
     }
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+    if (lane == 0) a.stats[h] = make_float2(m, s > 0.f ? 1.0f / s : 0.f);
 }
 
 // score[c] = sum over heads (in order) of exp(z - max) / sum; NaN off the candidates.
@@ -190,38 +211,12 @@ __global__ void __launch_bounds__(256) k_dec_vote(DecArgs a)
     a.scores[c] = sc;
 }
 
-// Key list of the step (one warp): sinks [0, min(n_sink, W_t)), the cached
-// selection's valid entries (inside [n_sink, W_t), increasing), the window [W_t, t].
-__global__ void __launch_bounds__(32) k_dec_list(DecArgs a)
-{
-    const int lane = threadIdx.x;
-    const int64_t W = window_start(a, a.t);
-    const int n_s = static_cast<int>(a.n_sink < W ? a.n_sink : W);
-    for (int i = lane; i < n_s; i += 32) a.list[i] = i;
-    int base = n_s;
-    int cnt = *a.sel_count;
-    cnt = cnt < 0 ? 0 : (cnt > a.k ? a.k : cnt);
-    for (int c0 = 0; c0 < cnt; c0 += 32) {
-        const int i = c0 + lane;
-        bool valid = false;
-        int32_t tok = 0;
-        if (i < cnt) {
-            tok = a.sel[i];
-            valid = tok >= a.n_sink && tok < W && (i == 0 || tok > a.sel[i - 1]);
-        }
-        const uint32_t b = __ballot_sync(0xFFFFFFFFu, valid);
-        if (valid) a.list[base + __popc(b & ((1u << lane) - 1u))] = tok;
-        base += __popc(b);
-    }
-    const int n_w = static_cast<int>(a.t - W + 1);
-    for (int i = lane; i < n_w; i += 32) a.list[base + i] = static_cast<int32_t>(W + i);
-    if (lane == 0) *a.list_n = base + n_w;
-}
-
-// Attention of the query over the listed keys, split over key chunks
-// (blockIdx.y): one warp per query head of KV head blockIdx.x, lane l holding
-// dimensions [4 l, 4 l + 4); online softmax in log2 units. Writes (max, sum,
-// unnormalised o) per (head, split).
+// Attention of the query over its keys, split over key chunks (blockIdx.y):
+// key i of the step is the sink i (i < n_s = min(n_sink, W_t)), then the
+// cached selection (produced by the top-k: ascending, inside [n_sink, W_a)
+// with W_a <= W_t), then the window [W_t, t]. One warp per query head of KV
+// head blockIdx.x, lane l holding dimensions [4 l, 4 l + 4); online softmax in
+// log2 units. Writes (max, sum, unnormalised o) per (head, split).
 __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16* __restrict__ q,
                                                   const uint2* __restrict__ k, const uint2* __restrict__ v)
 {
@@ -229,7 +224,11 @@ __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16
     const int lane = threadIdx.x & 31, hl = threadIdx.x >> 5;
     if (hl >= a.g) return;
     const int h = j * a.g + hl;
-    const int n = *a.list_n;
+    const int64_t W = window_start(a, a.t);
+    const int n_s = static_cast<int>(a.n_sink < W ? a.n_sink : W);
+    int n_sel = *a.sel_count;
+    n_sel = n_sel < 0 ? 0 : (n_sel > a.k ? a.k : n_sel);
+    const int n = n_s + n_sel + static_cast<int>(a.t - W + 1);
     const int per = (n + a.splits - 1) / a.splits;
     const int i0 = split * per, i1 = (i0 + per < n) ? i0 + per : n;
     const __nv_bfloat16* qh = q + h * kHeadDim + 4 * lane;
@@ -238,7 +237,8 @@ __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16
     float m = -INFINITY, l = 0.f, o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
 #pragma unroll 4
     for (int i = i0; i < i1; ++i) {
-        const int64_t row = (static_cast<int64_t>(a.list[i]) * a.Hkv + j) * 32 + lane;
+        const int64_t tok = i < n_s ? i : (i < n_s + n_sel ? a.sel[i - n_s] : W + (i - n_s - n_sel));
+        const int64_t row = (tok * a.Hkv + j) * 32 + lane;
         const uint2 kw = k[row];
         const uint2 vw = v[row];
         float s = q0 * bf16_lo(kw.x) + q1 * bf16_hi(kw.x) + q2 * bf16_lo(kw.y) + q3 * bf16_hi(kw.y);
@@ -298,12 +298,14 @@ size_t decode_ws_bytes(const Derived& d, int splits)
     off = align_up(off + static_cast<size_t>(d.Hq) * cap * sizeof(float), kAlign);  // z
     off = align_up(off + static_cast<size_t>(d.Hq) * sizeof(float2), kAlign);   // stats
     off = align_up(off + cap * sizeof(float), kAlign);                          // scores
-    off = align_up(off + (static_cast<size_t>(d.n_sink) + d.k + d.n_local + 1) * sizeof(int32_t) + 16, kAlign);
     off = align_up(off + static_cast<size_t>(d.Hq) * splits * 130 * sizeof(float), kAlign);
+    off = align_up(off + static_cast<size_t>(d.Hq) * ((cap + 127) / 128) * sizeof(float2), kAlign);  // zpart
+    off = align_up(off + (256 + 4) * sizeof(int32_t), kAlign);                                    // top-k hist, state
+    off = align_up(off + static_cast<size_t>(topk_max_chunks(d)) * sizeof(int2), kAlign);          // top-k counts
     return off;
 }
 
-constexpr int kDecSplits = 64;
+constexpr int kDecSplits = 128;
 
 int decode_splits() { return kDecSplits; }
 
@@ -339,18 +341,23 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
     a.z = reinterpret_cast<float*>(ws + take(static_cast<size_t>(d.Hq) * cap * sizeof(float)));
     a.stats = reinterpret_cast<float2*>(ws + take(static_cast<size_t>(d.Hq) * sizeof(float2)));
     a.scores = reinterpret_cast<float*>(ws + take(cap * sizeof(float)));
-    a.list = reinterpret_cast<int32_t*>(ws + take((static_cast<size_t>(d.n_sink) + d.k + d.n_local + 1) * sizeof(int32_t) + 16));
-    a.list_n = a.list + d.n_sink + d.k + d.n_local + 1;
     a.part = reinterpret_cast<float*>(ws + take(static_cast<size_t>(d.Hq) * kDecSplits * 130 * sizeof(float)));
+    a.zpart = reinterpret_cast<float2*>(ws + take(static_cast<size_t>(d.Hq) * ((cap + 127) / 128) * sizeof(float2)));
+    a.chunk = 128;  // 32 KB of staged logits for 32 heads: several CTAs per SM keep loads in flight
+    int32_t* tk_hist = reinterpret_cast<int32_t*>(ws + take((256 + 4) * sizeof(int32_t)));
+    int2* tk_counts = reinterpret_cast<int2*>(ws + take(static_cast<size_t>(topk_max_chunks(d)) * sizeof(int2)));
 
     const auto* qb = static_cast<const __nv_bfloat16*>(q);
     k_dec_gate<<<1, 256, 0, st>>>(a, qb);
     const int64_t n_cand = window_start(a, t) - d.n_sink;
     if (n_cand > 0) {
-        const unsigned blocks = static_cast<unsigned>(std::min<int64_t>((n_cand + 7) / 8, 152 * 16));
-        const size_t qsm = static_cast<size_t>(d.Hq) * kHeadDim * sizeof(float);
-        k_dec_logits<<<blocks, 256, qsm, st>>>(a, qb, static_cast<const uint2*>(k));
-        k_dec_stats<<<d.Hq, 256, 0, st>>>(a);
+        const int n_chunks = static_cast<int>((n_cand + a.chunk - 1) / a.chunk);
+        const size_t smem = (static_cast<size_t>(d.Hq) * kHeadDim + static_cast<size_t>(d.Hq) * a.chunk) * sizeof(float);
+        cudaError_t e0 = cudaFuncSetAttribute(k_dec_logits, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              static_cast<int>(smem));
+        if (e0 != cudaSuccess) return e0;
+        k_dec_logits<<<n_chunks, 128, smem, st>>>(a, qb, static_cast<const uint4*>(k));
+        k_dec_stats<<<(d.Hq + 7) / 8, 256, 0, st>>>(a, n_chunks);
         k_dec_vote<<<static_cast<unsigned>((t + 1 + 255) / 256), 256, 0, st>>>(a);
         // top-k of the one-unit table [t, t + 1] kept in the cache, gated on the retrieval flag
         Derived du = d;
@@ -358,15 +365,15 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
         du.B = 1;
         du.nb = d.N;
         const Units ut{a.units, a.units + 2, 0, d.N, 1, static_cast<int>(d.N)};
+        const TopkScratch scratch{tk_hist, tk_hist + 256, tk_counts, topk_max_chunks(du)};
         cudaError_t e = launch_topk(du, ut, static_cast<int>(t), static_cast<int>(t + 1), a.scores, a.sel,
-                                    a.sel_count, st, a.state + 2);
+                                    a.sel_count, st, a.state + 2, &scratch);
         if (e != cudaSuccess) return e;
     } else {
         // no candidates: the selection is empty whenever this step retrieves
         cudaError_t e = cudaMemsetAsync(a.sel_count, 0, sizeof(int32_t), st);
         if (e != cudaSuccess) return e;
     }
-    k_dec_list<<<1, 32, 0, st>>>(a);
     k_dec_attn<<<dim3(d.Hkv, kDecSplits), 32 * d.g, 0, st>>>(a, qb, static_cast<const uint2*>(k),
                                                               static_cast<const uint2*>(v));
     k_dec_combine<<<d.Hq, kHeadDim, 0, st>>>(a, static_cast<__nv_bfloat16*>(out));

@@ -347,7 +347,297 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
     if (threadIdx.x == 0) sel_count[u] = taken;
 }
 
+// ---- top-k over many candidates per unit: the same radix select and ordered
+// output as k_topk, spread over CTAs of kChunk candidates (grid y = unit).
+
+constexpr int kChunk = 8192;
+constexpr int kChunkThreads = 256;
+
+struct TopkState {
+    uint32_t prefix;  // bits of the k-th key fixed so far
+    int need;         // keys still to take at or below the prefix
+    int done;         // 1: the unit's output is already complete
+    int pad;
+};
+
+__device__ __forceinline__ bool unit_cands(const SelArgs& a, int ui, int* u, int64_t* lo, int64_t* hi)
+{
+    const int u_first = unit_lower_bound(a.ut, a.sc_begin);
+    const int u_end = unit_lower_bound(a.ut, a.sc_end);
+    *u = u_first + ui;
+    if (*u >= u_end) return false;
+    int anc;
+    int64_t s, e;
+    unit_range(a.ut, *u, &anc, &s, &e);
+    cand_range(a, s, lo, hi);
+    return true;
+}
+
+// Per unit: small candidate sets are written out directly; otherwise the
+// radix state starts (prefix 0, need k) and the histogram is cleared.
+__global__ void __launch_bounds__(256) k_topk_init(SelArgs a, int32_t* __restrict__ sel,
+                                                    int32_t* __restrict__ sel_count, int32_t* __restrict__ hist,
+                                                    TopkState* __restrict__ state)
+{
+    if (a.gate && !*a.gate) return;
+    int u;
+    int64_t lo, hi;
+    if (!unit_cands(a, blockIdx.x, &u, &lo, &hi)) return;
+    const int64_t n = hi - lo;
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[u * 256 + i] = 0;
+    if (n <= a.k) {
+        int32_t* out = sel + static_cast<int64_t>(u) * a.k;
+        for (int i = threadIdx.x; i < a.k; i += blockDim.x) out[i] = (i < n) ? static_cast<int32_t>(lo + i) : -1;
+        if (threadIdx.x == 0) {
+            sel_count[u] = static_cast<int32_t>(n);
+            state[u] = TopkState{0u, 0, 1, 0};
+        }
+    } else if (threadIdx.x == 0) {
+        state[u] = TopkState{0u, a.k, 0, 0};
+    }
+}
+
+// One radix pass: per-warp histograms of the digit at `shift` of the keys that
+// match the prefix, added into the unit's histogram.
+__global__ void __launch_bounds__(kChunkThreads) k_topk_hist(SelArgs a, const float* __restrict__ scores,
+                                                             int32_t* __restrict__ hist,
+                                                             const TopkState* __restrict__ state, int shift)
+{
+    __shared__ int wh[kChunkThreads / 32][256];
+    if (a.gate && !*a.gate) return;
+    int u;
+    int64_t lo, hi;
+    if (!unit_cands(a, blockIdx.y, &u, &lo, &hi)) return;
+    const TopkState stt = state[u];
+    if (stt.done) return;
+    const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * kChunk;
+    if (c0 >= hi) return;
+    const int64_t c1 = (c0 + kChunk < hi) ? c0 + kChunk : hi;
+    const int warp = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < (kChunkThreads / 32) * 256; i += blockDim.x) (&wh[0][0])[i] = 0;
+    __syncthreads();
+    const uint32_t mask = shift == 24 ? 0u : (0xFFFFFFFFu << (shift + 8));
+    const float* sc = scores + static_cast<int64_t>(u) * a.nb;
+    constexpr int kPer = kChunk / kChunkThreads;
+    uint32_t key[kPer];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+        const int64_t b = c0 + j * kChunkThreads + threadIdx.x;
+        key[j] = b < c1 ? float_key(sc[b]) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+        const int64_t b = c0 + j * kChunkThreads + threadIdx.x;
+        if (b < c1 && (key[j] & mask) == stt.prefix) atomicAdd(&wh[warp][(key[j] >> shift) & 255u], 1);
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) {
+        int c = 0;
+        for (int w = 0; w < kChunkThreads / 32; ++w) c += wh[w][i];
+        if (c) atomicAdd(&hist[u * 256 + i], c);
+    }
+}
+
+// The digit of the k-th largest key, from the unit's histogram; clears it.
+__global__ void __launch_bounds__(256) k_topk_pick(SelArgs a, int32_t* __restrict__ hist,
+                                                    TopkState* __restrict__ state, int shift)
+{
+    if (a.gate && !*a.gate) return;
+    int u;
+    int64_t lo, hi;
+    if (!unit_cands(a, blockIdx.x, &u, &lo, &hi)) return;
+    if (state[u].done) return;
+    __shared__ int h[256];
+    h[threadIdx.x] = hist[u * 256 + threadIdx.x];
+    hist[u * 256 + threadIdx.x] = 0;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        TopkState stt = state[u];
+        int need = stt.need, cum = 0, d = 255;
+        for (; d > 0; --d) {
+            if (cum + h[d] >= need) break;
+            cum += h[d];
+        }
+        stt.need = need - cum;
+        stt.prefix |= static_cast<uint32_t>(d) << shift;
+        state[u] = stt;
+    }
+}
+
+// Counts per chunk of the keys above the k-th key T and of the keys equal to it.
+__global__ void __launch_bounds__(kChunkThreads) k_topk_count(SelArgs a, const float* __restrict__ scores,
+                                                              const TopkState* __restrict__ state,
+                                                              int2* __restrict__ counts, int max_chunks)
+{
+    if (a.gate && !*a.gate) return;
+    int u;
+    int64_t lo, hi;
+    if (!unit_cands(a, blockIdx.y, &u, &lo, &hi)) return;
+    const TopkState stt = state[u];
+    if (stt.done) return;
+    const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * kChunk;
+    if (c0 >= hi) return;
+    const int64_t c1 = (c0 + kChunk < hi) ? c0 + kChunk : hi;
+    const float* sc = scores + static_cast<int64_t>(u) * a.nb;
+    int gt = 0, eq = 0;
+    for (int64_t b = c0 + threadIdx.x; b < c1; b += blockDim.x) {
+        const uint32_t key = float_key(sc[b]);
+        gt += key > stt.prefix;
+        eq += key == stt.prefix;
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        gt += __shfl_xor_sync(0xFFFFFFFFu, gt, o);
+        eq += __shfl_xor_sync(0xFFFFFFFFu, eq, o);
+    }
+    __shared__ int sg[kChunkThreads / 32], se[kChunkThreads / 32];
+    if ((threadIdx.x & 31) == 0) {
+        sg[threadIdx.x >> 5] = gt;
+        se[threadIdx.x >> 5] = eq;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int g = 0, e = 0;
+        for (int w = 0; w < kChunkThreads / 32; ++w) {
+            g += sg[w];
+            e += se[w];
+        }
+        counts[static_cast<int64_t>(u) * max_chunks + blockIdx.x] = make_int2(g, e);
+    }
+}
+
+// Per unit: output position and number of equal keys to take of every chunk
+// (the equal keys are taken lowest index first); the -1 padding and the count.
+__global__ void __launch_bounds__(32) k_topk_scan(SelArgs a, const TopkState* __restrict__ state,
+                                                   int2* __restrict__ counts, int max_chunks,
+                                                   int32_t* __restrict__ sel, int32_t* __restrict__ sel_count)
+{
+    if (a.gate && !*a.gate) return;
+    int u;
+    int64_t lo, hi;
+    if (!unit_cands(a, blockIdx.x, &u, &lo, &hi)) return;
+    const TopkState stt = state[u];
+    if (stt.done) return;
+    const int n_chunks = static_cast<int>((hi - lo + kChunk - 1) / kChunk);
+    int2* cu = counts + static_cast<int64_t>(u) * max_chunks;
+    __shared__ int s_total;
+    if (threadIdx.x == 0) {
+        int eq_before = 0, pos = 0;
+        for (int c = 0; c < n_chunks; ++c) {
+            const int2 ge = cu[c];
+            int take = stt.need - eq_before;
+            take = take < 0 ? 0 : (take > ge.y ? ge.y : take);
+            eq_before += ge.y;
+            cu[c] = make_int2(pos, take);
+            pos += ge.x + take;
+        }
+        s_total = pos;
+        sel_count[u] = pos;
+    }
+    __syncwarp();
+    int32_t* out = sel + static_cast<int64_t>(u) * a.k;
+    for (int i = s_total + threadIdx.x; i < a.k; i += 32) out[i] = -1;
+}
+
+// Ordered output of one chunk: every warp owns a contiguous segment (lane l
+// reads 4 consecutive keys per step), counts its picks, and after a scan over
+// the warps writes them in index order with warp prefix sums.
+__global__ void __launch_bounds__(kChunkThreads) k_topk_emit(SelArgs a, const float* __restrict__ scores,
+                                                             const TopkState* __restrict__ state,
+                                                             const int2* __restrict__ counts, int max_chunks,
+                                                             int32_t* __restrict__ sel)
+{
+    if (a.gate && !*a.gate) return;
+    int u;
+    int64_t lo, hi;
+    if (!unit_cands(a, blockIdx.y, &u, &lo, &hi)) return;
+    const TopkState stt = state[u];
+    if (stt.done) return;
+    const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * kChunk;
+    if (c0 >= hi) return;
+    const int64_t c1 = (c0 + kChunk < hi) ? c0 + kChunk : hi;
+    const int2 pt = counts[static_cast<int64_t>(u) * max_chunks + blockIdx.x];
+    const uint32_t T = stt.prefix;
+    const float* sc = scores + static_cast<int64_t>(u) * a.nb;
+    int32_t* out = sel + static_cast<int64_t>(u) * a.k;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int nw = kChunkThreads / 32;
+    const int64_t seg = kChunk / nw;
+    const int64_t w0 = c0 + seg * warp;
+    const int64_t w1 = (w0 + seg < c1) ? w0 + seg : c1;
+    int n_gt = 0, n_eq = 0;
+    for (int64_t b = w0 + 4 * lane; b < w1; b += 128)
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (b + j < w1) {
+                const uint32_t key = float_key(sc[b + j]);
+                n_gt += key > T;
+                n_eq += key == T;
+            }
+    for (int o = 16; o > 0; o >>= 1) {
+        n_gt += __shfl_xor_sync(0xFFFFFFFFu, n_gt, o);
+        n_eq += __shfl_xor_sync(0xFFFFFFFFu, n_eq, o);
+    }
+    __shared__ int s_take[nw], s_pos[nw];
+    if (lane == 0) {
+        s_take[warp] = n_eq;
+        s_pos[warp] = n_gt;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int eq_before = 0, pos = pt.x;
+        for (int w = 0; w < nw; ++w) {
+            const int e = s_take[w], g = s_pos[w];
+            int take = pt.y - eq_before;
+            take = take < 0 ? 0 : (take > e ? e : take);
+            eq_before += e;
+            s_take[w] = take;
+            s_pos[w] = pos;
+            pos += g + take;
+        }
+    }
+    __syncthreads();
+    int pos = s_pos[warp], take_eq = s_take[warp];
+    for (int64_t b = w0 + 4 * lane; b < w1; b += 128) {
+        uint32_t key[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) key[j] = (b + j < w1) ? float_key(sc[b + j]) : 0u;
+        int eq_l = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) eq_l += (b + j < w1) && key[j] == T;
+        int eq_inc = eq_l;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, eq_inc, o);
+            if (lane >= o) eq_inc += y;
+        }
+        const int eq_tot = __shfl_sync(0xFFFFFFFFu, eq_inc, 31);
+        int eq_rank = eq_inc - eq_l;
+        int pk[4], n_pk = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            pk[j] = 0;
+            if (b + j < w1) {
+                if (key[j] > T) pk[j] = 1;
+                else if (key[j] == T) pk[j] = (eq_rank++ < take_eq);
+            }
+            n_pk += pk[j];
+        }
+        int pk_inc = n_pk;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, pk_inc, o);
+            if (lane >= o) pk_inc += y;
+        }
+        int p = pos + pk_inc - n_pk;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            if (pk[j]) out[p++] = static_cast<int32_t>(b + j);
+        pos += __shfl_sync(0xFFFFFFFFu, pk_inc, 31);
+        take_eq -= (eq_tot < take_eq ? eq_tot : take_eq);
+    }
+}
+
 }  // namespace
+
+int topk_max_chunks(const Derived& d) { return static_cast<int>((d.nb + kChunk - 1) / kChunk); }
 
 cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
                           const float* reps, const float* fingerprints, const int32_t* unit_start,
@@ -393,7 +683,8 @@ cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t
 }
 
 cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_end, const float* scores,
-                        int32_t* sel, int32_t* sel_count, cudaStream_t st, const int32_t* gate)
+                        int32_t* sel, int32_t* sel_count, cudaStream_t st, const int32_t* gate,
+                        const TopkScratch* scratch)
 {
     SelArgs a{};
     a.gate = gate;
@@ -410,7 +701,22 @@ cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_
     a.sigma = d.sigma;
     const int max_units = sc_end - sc_begin;
     if (max_units <= 0) return cudaSuccess;
-    k_topk<<<max_units, kTopkThreads, 0, st>>>(a, scores, sel, sel_count);
+    if (!scratch || d.nb <= 8 * kChunk) {
+        k_topk<<<max_units, kTopkThreads, 0, st>>>(a, scores, sel, sel_count);
+        return cudaGetLastError();
+    }
+    // many candidates per unit: chunks of kChunk keys over the whole GPU
+    auto* state = reinterpret_cast<TopkState*>(scratch->state);
+    const int mc = scratch->max_chunks;
+    const dim3 grid(static_cast<unsigned>(mc), static_cast<unsigned>(max_units));
+    k_topk_init<<<max_units, 256, 0, st>>>(a, sel, sel_count, scratch->hist, state);
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        k_topk_hist<<<grid, kChunkThreads, 0, st>>>(a, scores, scratch->hist, state, shift);
+        k_topk_pick<<<max_units, 256, 0, st>>>(a, scratch->hist, state, shift);
+    }
+    k_topk_count<<<grid, kChunkThreads, 0, st>>>(a, scores, state, scratch->counts, mc);
+    k_topk_scan<<<max_units, 32, 0, st>>>(a, state, scratch->counts, mc, sel, sel_count);
+    k_topk_emit<<<grid, kChunkThreads, 0, st>>>(a, scores, state, scratch->counts, mc, sel);
     return cudaGetLastError();
 }
 

@@ -479,7 +479,10 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
     }
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    return launch_topk(d, a.ut, a.sc_begin, a.sc_end, a.scores, sel, sel_count, st);
+    const TopkScratch scratch{reinterpret_cast<int32_t*>(ws + lay.topk_hist),
+                              reinterpret_cast<int32_t*>(ws + lay.topk_state),
+                              reinterpret_cast<int2*>(ws + lay.topk_counts), topk_max_chunks(d)};
+    return launch_topk(d, a.ut, a.sc_begin, a.sc_end, a.scores, sel, sel_count, st, nullptr, &scratch);
 }
 
 }  // namespace scale
