@@ -78,7 +78,10 @@ def launches(w, selects: int = 1) -> dict:
     keys through a per-unit list)."""
     tok = w.block_size == 1
     build = (3 if tok else 4) + (1 if w.max_cluster_subchunks > 1 else 0)
-    select = 5 if tok else 4
+    # the top-k is one kernel, or 12 (init, 4 x (histogram, pick), count, scan,
+    # emit) for units of more than 64K candidates
+    topk = 12 if tok and w.n_blocks > 65536 else 1
+    select = (4 if tok else 3) + topk
     attend = 3 if tok else 1
     return {"build_reps": build, "select": select * selects, "attend": attend * selects,
             "total": build + (select + attend) * selects}
@@ -112,8 +115,8 @@ def profile_traffic():
     vals = {}
     with open(PROFILE_SUMMARY) as f:
         for line in f:
-            if ":" in line and line.strip().startswith("- "):
-                k, v = line.strip()[2:].split(":", 1)
+            if ": " in line and line.strip().startswith("- "):
+                k, v = line.strip()[2:].split(": ", 1)  # keys may hold a colon ("sha256[:16]")
                 vals[k.strip()] = v.strip()
     if vals.get("attn.cu sha256[:16]") != sha:
         return None

@@ -666,13 +666,10 @@ cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t
 
     const int upt = kLogitUnitRows / d.g;
     const size_t smem = (kLogitUnitRows * kHeadDim + kLogitBlocks * (kHeadDim + 1)) * sizeof(float);
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(k_logits, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(smem));
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    // set on every launch: the attribute belongs to the current device
+    cudaError_t e = cudaFuncSetAttribute(k_logits, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
     dim3 gl((max_units + upt - 1) / upt, static_cast<unsigned>((d.nb + kLogitBlocks - 1) / kLogitBlocks), d.Hkv);
     k_logits<<<gl, kLogitThreads, smem, st>>>(a, fingerprints, reps, logits);
     const int64_t rows = static_cast<int64_t>(max_units) * d.Hq;

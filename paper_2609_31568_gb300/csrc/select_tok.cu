@@ -403,16 +403,13 @@ template <int G>
 cudaError_t run_tok_passes(dim3 grid, int64_t rows, const CUtensorMap& tf, const CUtensorMap& tk,
                            const TokArgs& a, cudaStream_t st)
 {
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(k_tok_score<0, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(kSmemTok0));
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_tok_score<1, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     static_cast<int>(kSmemTok1));
-        if (e != cudaSuccess) return e;
-        attr = true;
-    }
+    // set on every launch: the attribute belongs to the current device
+    cudaError_t e = cudaFuncSetAttribute(k_tok_score<0, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kSmemTok0));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_tok_score<1, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kSmemTok1));
+    if (e != cudaSuccess) return e;
     k_tok_score<0, G><<<grid, kTokThreads, kSmemTok0, st>>>(tf, tk, a);
     k_tok_merge<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a);
     k_tok_score<1, G><<<grid, kTokThreads, kSmemTok1, st>>>(tf, tk, a);

@@ -411,8 +411,11 @@ def test_deterministic_bits():
                            y.view(torch.int32) if y.dtype == torch.float32 else y)
 
 
-def test_prefill_host_matches_device_path():
-    w, q, k, v, dev = inputs("gqa4-4k", **RAGGED)
+@pytest.mark.parametrize("over", [RAGGED, dict(block_size=1, top_k=64)])
+def test_prefill_host_matches_device_path(over):
+    """scale_prefill_host (host buffers in and out) gives the device path's
+    output bit for bit, at block level and at token level."""
+    w, q, k, v, dev = inputs("gqa4-4k", **over)
     for mode in (PER_CLUSTER, PER_SUB):
         p, buf = gpu_path(w, mode, dev, want_scores=False)
         arena = torch.empty(S.scale_prefill_host_arena_size(p, mode), dtype=torch.uint8, device="cuda")

@@ -74,3 +74,22 @@ def test_noalloc_refuses_problems_beyond_its_scratch():
         S.scale_build_reps_noalloc(p, small, small, small, small, ints, ints)
     assert e.value.rc == S.SCALE_ERR_WORKSPACE
     torch.cuda.synchronize()
+
+
+def test_noalloc_without_representatives_at_block_size_1():
+    """At block size 1 the representatives may be skipped (reps = NULL), as for
+    scale_build_reps; fingerprints and clusters are still written."""
+    pkg.build()
+    S.load()
+    w, q, k = _case("gqa4-4k", 9, block_size=1, top_k=64)
+    p = S.params_for(w)
+    _, fp, us, n = _outputs(S.params_for(w.replace(block_size=64)))
+    S.scale_build_reps_noalloc(p, q, k, None, fp, us, n)
+    ref = _outputs(S.params_for(w.replace(block_size=64)))
+    ws = torch.empty(S.scale_workspace_size(p, S.SCALE_MODE_PER_CLUSTER), dtype=torch.uint8, device="cuda")
+    S.scale_workspace_init(ws)
+    S.scale_build_reps(p, q, k, None, ref[1], ref[2], ref[3], ws)
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(fp.cpu().numpy(), ref[1].cpu().numpy(), rtol=0, atol=REPS_FP_ATOL)
+    assert torch.equal(n, ref[3])
+
