@@ -121,6 +121,24 @@ int scale_build_reps(const scale_params_t *p, const void *q, const void *k, floa
                      float *fingerprints, int32_t *unit_start, int32_t *n_units, void *ws,
                      size_t ws_bytes, scale_stream_t stream);
 
+/* Step (a) over the outer chunks that cover tokens [tok_begin, tok_end), for a
+ * caller that prefills chunk by chunk (Sec. III-B) and has the rows of later
+ * chunks not yet on the device. tok_begin is a multiple of the outer chunk
+ * length L_outer; tok_end is one too, or N. The ranges of a sequence are
+ * issued in order on one stream, starting at 0 and without gaps: each call
+ * appends its units to unit_start after the *n_units units of the earlier
+ * ranges (the first range, tok_begin = 0, starts the table), so that after the
+ * range ending at N the outputs equal those of scale_build_reps bit for bit.
+ * A call reads Q rows [tok_begin, tok_end) and K rows [tok_begin - B + 1,
+ * tok_end); it writes the fingerprints of the range's sub-chunks and the
+ * representatives of the blocks whose last token lies in the range (the range
+ * ending at N also writes the final, partial block). Arguments and errors as
+ * for scale_build_reps; a range that breaks the rules above returns
+ * SCALE_ERR_INVALID_ARG, and tok_begin == tok_end enqueues nothing. */
+int scale_build_reps_range(const scale_params_t *p, int64_t tok_begin, int64_t tok_end, const void *q,
+                           const void *k, float *reps, float *fingerprints, int32_t *unit_start,
+                           int32_t *n_units, void *ws, size_t ws_bytes, scale_stream_t stream);
+
 /* Step (a) without a workspace. The paper has no counterpart: this entry point
  * exists for callers that cannot allocate device memory for the library, such
  * as a host framework's plugin interface that hands over only input and output
@@ -233,6 +251,12 @@ int scale_build_reps_paged(const scale_params_t *p, const void *q, const scale_k
                            float *reps, float *fingerprints, int32_t *unit_start, int32_t *n_units,
                            void *ws, size_t ws_bytes, scale_stream_t stream);
 
+/* scale_build_reps_range with K read from a paged cache. */
+int scale_build_reps_range_paged(const scale_params_t *p, int64_t tok_begin, int64_t tok_end, const void *q,
+                                 const scale_kv_pages_t *kv, float *reps, float *fingerprints,
+                                 int32_t *unit_start, int32_t *n_units, void *ws, size_t ws_bytes,
+                                 scale_stream_t stream);
+
 /* scale_select_tokens with K read from a paged cache. */
 int scale_select_tokens_paged(const scale_params_t *p, int32_t mode, int64_t tok_begin,
                               int64_t tok_end, const scale_kv_pages_t *kv, const float *fingerprints,
@@ -291,7 +315,15 @@ int scale_retrieval_calls(const scale_params_t *p, int32_t mode, const int32_t *
  * back to out_host, and waits for `stream`. `arena` is a caller-owned device
  * buffer of scale_prefill_host_arena_size() bytes that holds the device copies,
  * the intermediate tensors and the workspace. Host buffers may be pageable;
- * pinned buffers make the copies asynchronous with respect to the host. */
+ * pinned buffers make the copies asynchronous with respect to the host.
+ * The call runs as chunked prefill does (Sec. III-B): in pieces of whole outer
+ * chunks (at most 64 pieces), each computed with the range calls
+ * (scale_build_reps_range, scale_select, scale_sparse_prefill) once its rows
+ * have arrived, while the next piece's rows are copied in and the previous
+ * piece's output is copied out on two streams of the call's own. When L or
+ * n_local is not a multiple of 128 it runs as one piece. The result equals the
+ * whole-sequence calls bit for bit. The call creates and releases those
+ * streams and their events itself. */
 int scale_prefill_host_arena_size(const scale_params_t *p, int32_t mode, size_t *bytes);
 int scale_prefill_host(const scale_params_t *p, int32_t mode, const void *q_host,
                        const void *k_host, const void *v_host, void *out_host, void *arena,

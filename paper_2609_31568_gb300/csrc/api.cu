@@ -3,6 +3,7 @@
 // end-to-end call that works from host buffers.
 #include <atomic>
 #include <cmath>
+#include <vector>
 
 #include "scale_internal.h"
 
@@ -165,6 +166,31 @@ Arena arena_layout(const Derived& d, int mode)
     return a;
 }
 
+// Two copy streams and the events of one scale_prefill_host call, released on
+// every return.
+struct CopyLanes {
+    cudaStream_t in = nullptr, out = nullptr;
+    std::vector<cudaEvent_t> events;
+    cudaError_t event(cudaEvent_t* ev)
+    {
+        const cudaError_t e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+        if (e == cudaSuccess) events.push_back(*ev);
+        return e;
+    }
+    ~CopyLanes()
+    {
+        // an early error return leaves no copy running into the caller's buffers
+        if (in) cudaStreamSynchronize(in);
+        if (out) cudaStreamSynchronize(out);
+        for (cudaEvent_t ev : events) cudaEventDestroy(ev);
+        if (in) cudaStreamDestroy(in);
+        if (out) cudaStreamDestroy(out);
+    }
+};
+
+// Upper bound on the pieces of one scale_prefill_host call.
+constexpr int kMaxHostPieces = 64;
+
 }  // namespace
 }  // namespace scale
 
@@ -205,17 +231,30 @@ int scale_workspace_init(void* ws, size_t ws_bytes, scale_stream_t stream)
     return cuda_status(cudaMemsetAsync(ws, 0, 256, stream));
 }
 
-static int build_reps_impl(const Derived& d, const void* q, const void* k, const KvPaging& pg,
-                           float* reps, float* fingerprints, int32_t* unit_start, int32_t* n_units,
-                           void* ws, size_t ws_bytes, scale_stream_t stream)
+// Outer chunks [*c_begin, *c_end) of the token range [tb, te): tb a multiple of
+// the outer chunk length, te one too or N.
+static int chunk_range(const Derived& d, int64_t tb, int64_t te, int* c_begin, int* c_end)
 {
-    int rc;
+    const int64_t L_outer = static_cast<int64_t>(d.per_outer) * d.L;
+    if (tb < 0 || te < tb || te > d.N || tb % L_outer || (te != d.N && te % L_outer))
+        return SCALE_ERR_INVALID_ARG;
+    *c_begin = static_cast<int>(tb / L_outer);
+    *c_end = static_cast<int>((te + L_outer - 1) / L_outer);
+    return SCALE_OK;
+}
+
+static int build_reps_impl(const Derived& d, int64_t tb, int64_t te, const void* q, const void* k,
+                           const KvPaging& pg, float* reps, float* fingerprints, int32_t* unit_start,
+                           int32_t* n_units, void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    int rc, c0, c1;
+    if ((rc = chunk_range(d, tb, te, &c0, &c1))) return rc;
     if (!device_ptr(q, 16) || !device_ptr(k, 16) || !(device_ptr(reps, 16) || (!reps && d.B == 1)) ||
         !device_ptr(fingerprints, 16) || !device_ptr(unit_start, 4) || !device_ptr(n_units, 4))
         return SCALE_ERR_INVALID_ARG;
     if ((rc = check_ws(d, ws, ws_bytes))) return rc;
-    return cuda_status(launch_build_reps(d, q, k, pg, reps, fingerprints, unit_start, n_units,
-                                         static_cast<uint8_t*>(ws), stream));
+    return cuda_status(launch_build_reps_range(d, q, k, pg, reps, fingerprints, unit_start, n_units, c0,
+                                               c1, static_cast<uint8_t*>(ws), stream));
 }
 
 int scale_build_reps(const scale_params_t* p, const void* q, const void* k, float* reps,
@@ -225,8 +264,19 @@ int scale_build_reps(const scale_params_t* p, const void* q, const void* k, floa
     Derived d;
     int rc = derive(p, &d);
     if (rc) return rc;
-    return build_reps_impl(d, q, k, contiguous(d), reps, fingerprints, unit_start, n_units, ws, ws_bytes,
-                           stream);
+    return build_reps_impl(d, 0, d.N, q, k, contiguous(d), reps, fingerprints, unit_start, n_units, ws,
+                           ws_bytes, stream);
+}
+
+int scale_build_reps_range(const scale_params_t* p, int64_t tok_begin, int64_t tok_end, const void* q,
+                           const void* k, float* reps, float* fingerprints, int32_t* unit_start,
+                           int32_t* n_units, void* ws, size_t ws_bytes, scale_stream_t stream)
+{
+    Derived d;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    return build_reps_impl(d, tok_begin, tok_end, q, k, contiguous(d), reps, fingerprints, unit_start,
+                           n_units, ws, ws_bytes, stream);
 }
 
 int scale_build_reps_paged(const scale_params_t* p, const void* q, const scale_kv_pages_t* kv, float* reps,
@@ -238,8 +288,22 @@ int scale_build_reps_paged(const scale_params_t* p, const void* q, const scale_k
     int rc = derive(p, &d);
     if (rc) return rc;
     if ((rc = check_pages(d, kv, &pg))) return rc;
-    return build_reps_impl(d, q, kv->k_pages, pg, reps, fingerprints, unit_start, n_units, ws, ws_bytes,
-                           stream);
+    return build_reps_impl(d, 0, d.N, q, kv->k_pages, pg, reps, fingerprints, unit_start, n_units, ws,
+                           ws_bytes, stream);
+}
+
+int scale_build_reps_range_paged(const scale_params_t* p, int64_t tok_begin, int64_t tok_end, const void* q,
+                                 const scale_kv_pages_t* kv, float* reps, float* fingerprints,
+                                 int32_t* unit_start, int32_t* n_units, void* ws, size_t ws_bytes,
+                                 scale_stream_t stream)
+{
+    Derived d;
+    KvPaging pg;
+    int rc = derive(p, &d);
+    if (rc) return rc;
+    if ((rc = check_pages(d, kv, &pg))) return rc;
+    return build_reps_impl(d, tok_begin, tok_end, q, kv->k_pages, pg, reps, fingerprints, unit_start,
+                           n_units, ws, ws_bytes, stream);
 }
 
 int scale_select(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64_t tok_end,
@@ -427,12 +491,8 @@ int scale_prefill_host(const scale_params_t* p, int32_t mode, const void* q_host
     const Arena A = arena_layout(d, mode);
     if (arena_bytes < A.total) return SCALE_ERR_WORKSPACE;
     uint8_t* base = static_cast<uint8_t*>(arena);
-    const size_t qb = static_cast<size_t>(d.N) * d.Hq * kHeadDim * 2;
-    const size_t kb = static_cast<size_t>(d.N) * d.Hkv * kHeadDim * 2;
-    cudaError_t e = cudaMemcpyAsync(base + A.q, q_host, qb, cudaMemcpyHostToDevice, stream);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(base + A.k, k_host, kb, cudaMemcpyHostToDevice, stream);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(base + A.v, v_host, kb, cudaMemcpyHostToDevice, stream);
-    if (e != cudaSuccess) return SCALE_ERR_CUDA;
+    const size_t q_row = static_cast<size_t>(d.Hq) * kHeadDim * 2;
+    const size_t kv_row_b = static_cast<size_t>(d.Hkv) * kHeadDim * 2;
     void* ws = base + A.ws;
     const size_t wsb = arena_bytes - A.ws;
     auto* reps = d.B == 1 ? nullptr : reinterpret_cast<float*>(base + A.reps);
@@ -441,15 +501,68 @@ int scale_prefill_host(const scale_params_t* p, int32_t mode, const void* q_host
     auto* nu = reinterpret_cast<int32_t*>(base + A.n_units);
     auto* sel = reinterpret_cast<int32_t*>(base + A.sel);
     auto* cnt = reinterpret_cast<int32_t*>(base + A.sel_count);
+
+    // Pieces of whole outer chunks. Piece p computes once its own rows are on
+    // the device (the rows before it arrived first, on the same copy stream);
+    // its output rows go back while piece p + 1 computes. Every row a piece
+    // reads lies before its end when L and n_local are multiples of 128 (the
+    // causal window's 128-row tiles then end at the query block's end);
+    // otherwise a tile may reach rows that the next piece's copy is writing,
+    // and the call runs as one piece.
+    const int n_chunks = outer_chunks(d);
+    const bool split = d.L % 128 == 0 && d.n_local % 128 == 0;
+    int per_piece = split ? (n_chunks + kMaxHostPieces - 1) / kMaxHostPieces : n_chunks;
+    const int pieces = (n_chunks + per_piece - 1) / per_piece;
+    const int64_t L_outer = static_cast<int64_t>(d.per_outer) * d.L;
+
+    CopyLanes lanes;
+    cudaEvent_t ev_start, ev_end;
+    cudaError_t e = cudaStreamCreateWithFlags(&lanes.in, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&lanes.out, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = lanes.event(&ev_start);
+    if (e == cudaSuccess) e = lanes.event(&ev_end);
+    if (e == cudaSuccess) e = cudaEventRecord(ev_start, stream);  // the arena's earlier users
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(lanes.in, ev_start, 0);
+    if (e != cudaSuccess) return SCALE_ERR_CUDA;
     if ((rc = scale_workspace_init(ws, wsb, stream))) return rc;
-    if ((rc = scale_build_reps(p, base + A.q, base + A.k, reps, fp, us, nu, ws, wsb, stream))) return rc;
-    rc = d.B == 1 ? scale_select_tokens(p, mode, 0, d.N, base + A.k, fp, us, nu, sel, cnt, nullptr, ws, wsb, stream)
-                  : scale_select(p, mode, 0, d.N, reps, fp, us, nu, sel, cnt, nullptr, ws, wsb, stream);
-    if (rc) return rc;
-    if ((rc = scale_sparse_prefill(p, mode, 0, d.N, base + A.q, base + A.k, base + A.v, us, nu, sel,
-                                   cnt, base + A.out, ws, wsb, stream)))
-        return rc;
-    e = cudaMemcpyAsync(out_host, base + A.out, qb, cudaMemcpyDeviceToHost, stream);
+
+    for (int pc = 0; pc < pieces; ++pc) {
+        const int64_t t0 = static_cast<int64_t>(pc) * per_piece * L_outer;
+        const int64_t t1 = (pc + 1 == pieces) ? d.N : t0 + per_piece * L_outer;
+        const size_t rows = static_cast<size_t>(t1 - t0);
+        cudaEvent_t ev_in, ev_done;
+        e = lanes.event(&ev_in);
+        if (e == cudaSuccess) e = lanes.event(&ev_done);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(base + A.q + t0 * q_row, static_cast<const uint8_t*>(q_host) + t0 * q_row,
+                                rows * q_row, cudaMemcpyHostToDevice, lanes.in);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(base + A.k + t0 * kv_row_b, static_cast<const uint8_t*>(k_host) + t0 * kv_row_b,
+                                rows * kv_row_b, cudaMemcpyHostToDevice, lanes.in);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(base + A.v + t0 * kv_row_b, static_cast<const uint8_t*>(v_host) + t0 * kv_row_b,
+                                rows * kv_row_b, cudaMemcpyHostToDevice, lanes.in);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_in, lanes.in);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(stream, ev_in, 0);
+        if (e != cudaSuccess) return SCALE_ERR_CUDA;
+        if ((rc = scale_build_reps_range(p, t0, t1, base + A.q, base + A.k, reps, fp, us, nu, ws, wsb, stream)))
+            return rc;
+        rc = d.B == 1 ? scale_select_tokens(p, mode, t0, t1, base + A.k, fp, us, nu, sel, cnt, nullptr, ws, wsb,
+                                            stream)
+                      : scale_select(p, mode, t0, t1, reps, fp, us, nu, sel, cnt, nullptr, ws, wsb, stream);
+        if (rc) return rc;
+        if ((rc = scale_sparse_prefill(p, mode, t0, t1, base + A.q, base + A.k, base + A.v, us, nu, sel, cnt,
+                                       base + A.out, ws, wsb, stream)))
+            return rc;
+        e = cudaEventRecord(ev_done, stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(lanes.out, ev_done, 0);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(static_cast<uint8_t*>(out_host) + t0 * q_row, base + A.out + t0 * q_row,
+                                rows * q_row, cudaMemcpyDeviceToHost, lanes.out);
+        if (e != cudaSuccess) return SCALE_ERR_CUDA;
+    }
+    e = cudaEventRecord(ev_end, lanes.out);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(stream, ev_end, 0);
     if (e != cudaSuccess) return SCALE_ERR_CUDA;
     int32_t st = 0;
     if ((rc = scale_get_device_status(ws, stream, &st))) return rc;

@@ -33,13 +33,14 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p)
 // Representative key of block b for every KV head: the mean of the block's
 // keys. One CTA per block; thread c owns elements [8c, 8c+8) of the token row
 // (H_kv * 128 elements), so every token row is read as one coalesced span.
+// Grid: the blocks [b_base, b_base + gridDim.x).
 __global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k, KvPaging pg, int64_t N,
-                                                      int row_chunks, int B, int64_t nb,
+                                                      int row_chunks, int B, int64_t nb, int64_t b_base,
                                                       float* __restrict__ reps)
 {
     const int c = threadIdx.x;
     if (c >= row_chunks) return;
-    const int64_t b = blockIdx.x;
+    const int64_t b = b_base + blockIdx.x;
     const int64_t t0 = b * B;
     const int64_t t1 = (t0 + B < N) ? t0 + B : N;
     float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
@@ -69,12 +70,12 @@ __global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k
 }
 
 // Partial sums of the multi-head queries of sub-chunk i over token split s
-// (split_len tokens). Grid (M, splits).
+// (split_len tokens). Grid (sub-chunks [m0, m0 + gridDim.x), splits).
 __global__ void __launch_bounds__(512) k_fp_partial(const uint4* __restrict__ q, int64_t N, int D8,
-                                                     int L, int split_len, int splits,
+                                                     int L, int split_len, int splits, int64_t m0,
                                                      float* __restrict__ partial)
 {
-    const int64_t i = blockIdx.x;
+    const int64_t i = m0 + blockIdx.x;
     const int s = blockIdx.y;
     const int64_t sc0 = i * L;
     const int64_t sc1 = (sc0 + L < N) ? sc0 + L : N;
@@ -117,14 +118,15 @@ __device__ float block_sum(float v, float* red)
     return t;
 }
 
-// v_i = (sum of the partials in split order) / |X_i|, and ||v_i||_2.
+// v_i = (sum of the partials in split order) / |X_i|, and ||v_i||_2, for
+// i in [m0, m0 + gridDim.x).
 __global__ void __launch_bounds__(512) k_fp_finalize(const float* __restrict__ partial, int D,
-                                                      int splits, int L, int64_t N,
+                                                      int splits, int L, int64_t N, int64_t m0,
                                                       float* __restrict__ fp,
                                                       float* __restrict__ norms)
 {
     __shared__ float red[32];
-    const int64_t i = blockIdx.x;
+    const int64_t i = m0 + blockIdx.x;
     const int64_t cnt = ((i + 1) * L < N ? (i + 1) * L : N) - i * L;
     const float inv_cnt = 1.0f / static_cast<float>(cnt);
     float ss = 0.f;
@@ -140,11 +142,12 @@ __global__ void __launch_bounds__(512) k_fp_finalize(const float* __restrict__ p
 }
 
 // gram[i][d] = cos(v_i, v_{i+d}) = v~_i . v~_{i+d} for 1 <= d < S_max and i+d
-// in the same outer chunk; 0 when either norm is 0. One warp per (i, d).
+// in the same outer chunk; 0 when either norm is 0. One warp per (i, d);
+// one CTA per i in [m0, m0 + gridDim.x).
 __global__ void k_gram(const float* __restrict__ fp, const float* __restrict__ norms, int D, int M,
-                       int S_max, int per_outer, float* __restrict__ gram)
+                       int S_max, int per_outer, int m0, float* __restrict__ gram)
 {
-    const int i = blockIdx.x;
+    const int i = m0 + static_cast<int>(blockIdx.x);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nw = blockDim.x >> 5;
     const int chunk_end = min(M, (i / per_outer + 1) * per_outer);
@@ -191,19 +194,23 @@ __device__ int block_exclusive_scan(int f, int* sh, int* total)
     return excl;
 }
 
-// Algorithm 1 in each outer chunk (one thread per chunk walks its sub-chunks:
-// the anchor a admits j while cos(v_a, v_j) >= theta and |C_a| < S_max), then
-// one block compacts the anchor flags into unit_start and n_units.
+// Algorithm 1 in the outer chunks [c_begin, c_end) (one thread per chunk walks
+// its sub-chunks: the anchor a admits j while cos(v_a, v_j) >= theta and
+// |C_a| < S_max), then one block compacts the anchor flags of those chunks
+// into unit_start, after the *n_units units of the chunks before c_begin.
 __global__ void __launch_bounds__(1024) k_cluster(const float* __restrict__ gram, int M, int S_max,
-                                                  int per_outer, float theta,
+                                                  int per_outer, float theta, int c_begin, int c_end,
                                                   int32_t* __restrict__ flag,
                                                   int32_t* __restrict__ unit_start,
                                                   int32_t* __restrict__ n_units)
 {
     __shared__ int sh[40];
     const bool always = theta <= -1.0f;
-    const int n_chunks = (M + per_outer - 1) / per_outer;
-    for (int c = threadIdx.x; c < n_chunks; c += blockDim.x) {
+    // read before the first barrier; thread 0 rewrites it after the last
+    int offset = c_begin == 0 ? 0 : *n_units;
+    const int m_begin = c_begin * per_outer;
+    const int m_end = min(M, c_end * per_outer);
+    for (int c = c_begin + static_cast<int>(threadIdx.x); c < c_end; c += blockDim.x) {
         const int c0 = c * per_outer;
         const int c1 = min(M, c0 + per_outer);
         int a = c0;
@@ -221,10 +228,9 @@ __global__ void __launch_bounds__(1024) k_cluster(const float* __restrict__ gram
         }
     }
     __syncthreads();
-    int offset = 0;
-    for (int base = 0; base < M; base += blockDim.x) {
+    for (int base = m_begin; base < m_end; base += blockDim.x) {
         const int i = base + threadIdx.x;
-        const int f = (i < M) ? flag[i] : 0;
+        const int f = (i < m_end) ? flag[i] : 0;
         int total;
         const int excl = block_exclusive_scan(f, sh, &total);
         if (f) unit_start[offset + excl] = i;
@@ -236,36 +242,62 @@ __global__ void __launch_bounds__(1024) k_cluster(const float* __restrict__ gram
 
 }  // namespace
 
-cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, const KvPaging& pg,
-                              float* reps, float* fingerprints, int32_t* unit_start, int32_t* n_units,
-                              uint8_t* ws, cudaStream_t st)
+int outer_chunks(const Derived& d)
 {
+    return static_cast<int>((d.M + d.per_outer - 1) / d.per_outer);
+}
+
+cudaError_t launch_build_reps_range(const Derived& d, const void* q, const void* k, const KvPaging& pg,
+                                    float* reps, float* fingerprints, int32_t* unit_start,
+                                    int32_t* n_units, int c_begin, int c_end, uint8_t* ws,
+                                    cudaStream_t st)
+{
+    if (c_begin < 0 || c_end > outer_chunks(d) || c_begin >= c_end) return cudaSuccess;
     const WsLayout lay = ws_layout(d);
     float* partial = reinterpret_cast<float*>(ws + lay.fp_partial);
     float* norms = reinterpret_cast<float*>(ws + lay.norms);
     float* gram = reinterpret_cast<float*>(ws + lay.gram);
     int32_t* flag = reinterpret_cast<int32_t*>(ws + lay.anchor);
 
+    // Tokens [t0, t1) and sub-chunks [m0, m1) of the chunks. A block belongs to
+    // the range holding its last token, so every key it averages is present
+    // once the chunks up to this range are.
+    const int64_t L_outer = static_cast<int64_t>(d.per_outer) * d.L;
+    const int64_t t0 = c_begin * L_outer;
+    const int64_t t1 = c_end * L_outer < d.N ? c_end * L_outer : d.N;
+    const int64_t m0 = static_cast<int64_t>(c_begin) * d.per_outer;
+    const int64_t m1 = static_cast<int64_t>(c_end) * d.per_outer < d.M ? static_cast<int64_t>(c_end) * d.per_outer
+                                                                         : d.M;
+    const int64_t b0 = t0 / d.B;
+    const int64_t b1 = t1 == d.N ? d.nb : t1 / d.B;
+
     const int row_chunks = d.Hkv * (kHeadDim / 8);
-    if (reps)  // block size 1 may skip them: token-level selection reads K itself
-        k_block_reps<<<static_cast<unsigned>(d.nb), row_chunks, 0, st>>>(
-            static_cast<const uint4*>(k), pg, d.N, row_chunks, d.B, d.nb, reps);
+    if (reps && b1 > b0)  // block size 1 may skip them: token-level selection reads K itself
+        k_block_reps<<<static_cast<unsigned>(b1 - b0), row_chunks, 0, st>>>(
+            static_cast<const uint4*>(k), pg, d.N, row_chunks, d.B, d.nb, b0, reps);
 
     const int D8 = d.D / 8;
     const int split_len = (d.L + d.fp_splits - 1) / d.fp_splits;
-    k_fp_partial<<<dim3(static_cast<unsigned>(d.M), d.fp_splits), D8 < 512 ? D8 : 512, 0, st>>>(
-        static_cast<const uint4*>(q), d.N, D8, d.L, split_len, d.fp_splits, partial);
-    k_fp_finalize<<<static_cast<unsigned>(d.M), 512, 0, st>>>(partial, d.D, d.fp_splits, d.L, d.N,
-                                                               fingerprints, norms);
+    const unsigned nm = static_cast<unsigned>(m1 - m0);
+    k_fp_partial<<<dim3(nm, d.fp_splits), D8 < 512 ? D8 : 512, 0, st>>>(
+        static_cast<const uint4*>(q), d.N, D8, d.L, split_len, d.fp_splits, m0, partial);
+    k_fp_finalize<<<nm, 512, 0, st>>>(partial, d.D, d.fp_splits, d.L, d.N, m0, fingerprints, norms);
     if (d.S_max > 1) {
         const int warps = d.S_max - 1 < 16 ? d.S_max - 1 : 16;
-        k_gram<<<static_cast<unsigned>(d.M), 32 * warps, 0, st>>>(fingerprints, norms, d.D,
-                                                                  static_cast<int>(d.M), d.S_max,
-                                                                  d.per_outer, gram);
+        k_gram<<<nm, 32 * warps, 0, st>>>(fingerprints, norms, d.D, static_cast<int>(d.M), d.S_max,
+                                          d.per_outer, static_cast<int>(m0), gram);
     }
-    k_cluster<<<1, 1024, 0, st>>>(gram, static_cast<int>(d.M), d.S_max, d.per_outer, d.theta, flag,
-                                  unit_start, n_units);
+    k_cluster<<<1, 1024, 0, st>>>(gram, static_cast<int>(d.M), d.S_max, d.per_outer, d.theta, c_begin,
+                                  c_end, flag, unit_start, n_units);
     return cudaGetLastError();
+}
+
+cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, const KvPaging& pg,
+                              float* reps, float* fingerprints, int32_t* unit_start, int32_t* n_units,
+                              uint8_t* ws, cudaStream_t st)
+{
+    return launch_build_reps_range(d, q, k, pg, reps, fingerprints, unit_start, n_units, 0,
+                                   outer_chunks(d), ws, st);
 }
 
 }  // namespace scale

@@ -155,6 +155,13 @@ __device__ __forceinline__ void record_status(int32_t* status, int32_t code)
 cudaError_t launch_build_reps(const Derived& d, const void* q, const void* k, const KvPaging& pg,
                               float* reps, float* fingerprints, int32_t* unit_start, int32_t* n_units,
                               uint8_t* ws, cudaStream_t st);
+// Step (a) over the outer chunks [c_begin, c_end), appending their units to
+// unit_start after the *n_units units of the chunks before c_begin.
+cudaError_t launch_build_reps_range(const Derived& d, const void* q, const void* k, const KvPaging& pg,
+                                    float* reps, float* fingerprints, int32_t* unit_start,
+                                    int32_t* n_units, int c_begin, int c_end, uint8_t* ws,
+                                    cudaStream_t st);
+int outer_chunks(const Derived& d);
 cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
                           const float* reps, const float* fingerprints, const int32_t* unit_start,
                           const int32_t* n_units, int32_t* sel_blocks, int32_t* sel_count,

@@ -124,6 +124,8 @@ def load() -> ctypes.CDLL:
             "scale_select": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, sz, P],
             "scale_select_tokens": [pp, i32, i64, i64, P, P, P, P, P, P, P, P, sz, P],
             "scale_build_reps_paged": [pp, P, kp, P, P, P, P, P, sz, P],
+            "scale_build_reps_range": [pp, i64, i64, P, P, P, P, P, P, P, sz, P],
+            "scale_build_reps_range_paged": [pp, i64, i64, P, kp, P, P, P, P, P, sz, P],
             "scale_select_tokens_paged": [pp, i32, i64, i64, kp, P, P, P, P, P, P, P, sz, P],
             "scale_sparse_prefill_paged": [pp, i32, i64, i64, P, kp, P, P, P, P, P, P, sz, P],
             "scale_decode_cache_size": [pp, ctypes.POINTER(sz)],
@@ -213,6 +215,14 @@ def scale_build_reps(p, q, k, reps, fingerprints, unit_start, n_units, ws, strea
         _ptr(n_units), _ptr(ws), _nbytes(ws), _stream(stream)))
 
 
+def scale_build_reps_range(p, tok_begin, tok_end, q, k, reps, fingerprints, unit_start, n_units, ws,
+                           stream=None) -> None:
+    """Step (a) over the outer chunks covering [tok_begin, tok_end); ranges go in order from 0."""
+    _check("scale_build_reps_range", load().scale_build_reps_range(
+        ctypes.byref(p), tok_begin, tok_end, _ptr(q), _ptr(k), _ptr(reps), _ptr(fingerprints),
+        _ptr(unit_start), _ptr(n_units), _ptr(ws), _nbytes(ws), _stream(stream)))
+
+
 def scale_build_reps_noalloc(p, q, k, reps, fingerprints, unit_start, n_units, stream=None) -> None:
     """Step (a) with the library's fixed scratch array instead of a workspace."""
     _check("scale_build_reps_noalloc", load().scale_build_reps_noalloc(
@@ -249,6 +259,13 @@ def scale_build_reps_paged(p, q, kv: ScaleKvPages, reps, fingerprints, unit_star
     _check("scale_build_reps_paged", load().scale_build_reps_paged(
         ctypes.byref(p), _ptr(q), ctypes.byref(kv), _ptr(reps), _ptr(fingerprints), _ptr(unit_start),
         _ptr(n_units), _ptr(ws), _nbytes(ws), _stream(stream)))
+
+
+def scale_build_reps_range_paged(p, tok_begin, tok_end, q, kv: ScaleKvPages, reps, fingerprints,
+                                 unit_start, n_units, ws, stream=None) -> None:
+    _check("scale_build_reps_range_paged", load().scale_build_reps_range_paged(
+        ctypes.byref(p), tok_begin, tok_end, _ptr(q), ctypes.byref(kv), _ptr(reps), _ptr(fingerprints),
+        _ptr(unit_start), _ptr(n_units), _ptr(ws), _nbytes(ws), _stream(stream)))
 
 
 def scale_select_tokens_paged(p, mode, tok_begin, tok_end, kv: ScaleKvPages, fingerprints, unit_start,

@@ -21,6 +21,8 @@ PER_CLUSTER, PER_SUB = S.SCALE_MODE_PER_CLUSTER, S.SCALE_MODE_PER_SUBCHUNK
 
 # Small cases that span several tiles and end in ragged pieces.
 RAGGED = dict(n_tokens=3000, block_size=48, n_sink=40, n_local=100, top_k=6)
+# Ragged too, with a window of whole 128-row tiles: the host call runs in pieces.
+RAGGED_PIECES = dict(n_tokens=3000, block_size=48, n_sink=40, n_local=128, top_k=6)
 GQA_SMALL = dict(n_tokens=8192 + 333, sub_chunk=512, max_cluster_subchunks=4, outer_chunk=2048,
                  top_k=8)
 
@@ -411,10 +413,12 @@ def test_deterministic_bits():
                            y.view(torch.int32) if y.dtype == torch.float32 else y)
 
 
-@pytest.mark.parametrize("over", [RAGGED, dict(block_size=1, top_k=64)])
+@pytest.mark.parametrize("over", [RAGGED, RAGGED_PIECES, dict(block_size=1, top_k=64)])
 def test_prefill_host_matches_device_path(over):
     """scale_prefill_host (host buffers in and out) gives the device path's
-    output bit for bit, at block level and at token level."""
+    output bit for bit, at block level and at token level, whether it runs as
+    one piece (a window that is not whole tiles) or in pieces of outer chunks
+    overlapped with the copies."""
     w, q, k, v, dev = inputs("gqa4-4k", **over)
     for mode in (PER_CLUSTER, PER_SUB):
         p, buf = gpu_path(w, mode, dev, want_scores=False)
@@ -422,6 +426,53 @@ def test_prefill_host_matches_device_path(over):
         out = np.empty((w.n_tokens, w.num_q_heads, w.head_dim), np.uint16)
         S.scale_prefill_host(p, mode, q, k, v, out, arena)
         assert np.array_equal(out, buf.out.view(torch.int16).cpu().numpy().view(np.uint16))
+
+
+@pytest.mark.parametrize("over", [RAGGED_PIECES, dict(block_size=1, top_k=64)])
+def test_range_calls_read_no_row_past_the_range(over):
+    """Chunked prefill (Sec. III-B) with the range calls: the device copies of
+    Q, K and V start as NaN and the rows of each outer chunk arrive just before
+    its calls. A read of any row past the range would put NaN into the
+    representatives, the fingerprints, the scores or (through P = 0 times a NaN
+    value row) the output; the results must equal the whole-sequence calls bit
+    for bit, including the unit table that the ranges build by appending."""
+    w, q, k, v, dev = inputs("gqa4-4k", **over)
+    for mode in (PER_CLUSTER, PER_SUB):
+        p, whole = gpu_path(w, mode, dev, want_scores=False)
+        late = [torch.full_like(x, float("nan")) for x in dev]
+        buf = S.allocate(p, mode)
+        buf.out.fill_(float("nan"))  # every row must be written by its own range
+        for t0 in range(0, w.n_tokens, w.outer_chunk):
+            t1 = min(w.n_tokens, t0 + w.outer_chunk)
+            for dst, src in zip(late, dev):
+                dst[t0:t1].copy_(src[t0:t1])
+            S.scale_build_reps_range(p, t0, t1, late[0], late[1], buf.reps, buf.fingerprints,
+                                     buf.unit_start, buf.n_units, buf.ws)
+            S.select(p, mode, t0, t1, late[1], buf)
+            S.scale_sparse_prefill(p, mode, t0, t1, *late, buf.unit_start, buf.n_units, buf.sel_blocks,
+                                   buf.sel_count, buf.out, buf.ws)
+        torch.cuda.synchronize()
+        assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
+        n = unit_count(whole, mode, w)
+        assert int(buf.n_units.item()) == int(whole.n_units.item())
+        assert torch.equal(buf.unit_start, whole.unit_start)
+        assert torch.equal(buf.fingerprints.view(torch.int32), whole.fingerprints.view(torch.int32))
+        if whole.reps is not None:
+            assert torch.equal(buf.reps.view(torch.int32), whole.reps.view(torch.int32))
+        assert torch.equal(buf.sel_count[:n], whole.sel_count[:n])
+        assert torch.equal(buf.sel_blocks[:n], whole.sel_blocks[:n])
+        assert torch.equal(buf.out.view(torch.int16), whole.out.view(torch.int16))
+
+
+def test_range_calls_reject_ranges_off_the_outer_chunks():
+    w, q, k, v, dev = inputs("gqa4-4k")
+    p = S.params_for(w)
+    buf = S.allocate(p, PER_CLUSTER)
+    for t0, t1 in ((256, 2048), (0, 1000), (1024, 512), (0, w.n_tokens + 1024)):
+        with pytest.raises(S.ScaleError) as e:
+            S.scale_build_reps_range(p, t0, t1, dev[0], dev[1], buf.reps, buf.fingerprints,
+                                     buf.unit_start, buf.n_units, buf.ws)
+        assert e.value.rc == S.SCALE_ERR_INVALID_ARG
 
 
 def test_wait_timeout_is_reported_and_context_survives():
