@@ -45,6 +45,8 @@ def parse_args():
     ap.add_argument("--mode", choices=["cluster", "subchunk"], default="cluster")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-chunk-loop", action="store_true",
+                    help="skip timing the per-outer-chunk loop of range calls alongside")
     ap.add_argument("--no-baseline-mode", action="store_true",
                     help="skip timing the per-sub-chunk selection mode alongside")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -72,10 +74,11 @@ def load_peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sustained=1700.0, source="fallback")
 
 
-def launches(w, selects: int = 1) -> dict:
-    """Kernels each call of the path launches for workload w (block size 1
-    skips the representatives, scores in four kernels and gathers the distant
-    keys through a per-unit list)."""
+def launches(w, selects: int = 1, builds: int = 1) -> dict:
+    """Kernels the path launches for workload w with `builds` step-(a) calls and
+    `selects` select + attend calls (block size 1 skips the representatives,
+    scores in four kernels and gathers the distant keys through a per-unit
+    list)."""
     tok = w.block_size == 1
     build = (3 if tok else 4) + (1 if w.max_cluster_subchunks > 1 else 0)
     # the top-k is one kernel, or 12 (init, 4 x (histogram, pick), count, scan,
@@ -83,8 +86,8 @@ def launches(w, selects: int = 1) -> dict:
     topk = 12 if tok and w.n_blocks > 65536 else 1
     select = (4 if tok else 3) + topk
     attend = 3 if tok else 1
-    return {"build_reps": build, "select": select * selects, "attend": attend * selects,
-            "total": build + (select + attend) * selects}
+    return {"build_reps": build * builds, "select": select * selects, "attend": attend * selects,
+            "total": build * builds + (select + attend) * selects}
 
 
 def key_counts(w, unit_start, n_units, sel, cnt, per_subchunk):
@@ -416,6 +419,51 @@ def run_scale(args):
                               "retrieval_calls": calls2, "units": n2}
         del buf2
 
+    if not args.no_chunk_loop and rank == 0:
+        # Chunked prefill as Algorithm 2 orders it: per outer chunk, step (a)
+        # over the chunk's range, then its selection and attention.
+        chunks = [(t0, min(w.n_tokens, t0 + w.outer_chunk)) for t0 in range(0, w.n_tokens, w.outer_chunk)]
+
+        def chunk_step():
+            for t0, t1 in chunks:
+                if kv is not None:
+                    S.scale_build_reps_range_paged(p, t0, t1, dev[0], kv, buf.reps, buf.fingerprints,
+                                                   buf.unit_start, buf.n_units, buf.ws, stream)
+                    if w.block_size == 1:
+                        S.scale_select_tokens_paged(p, mode, t0, t1, kv, buf.fingerprints, buf.unit_start,
+                                                    buf.n_units, buf.sel_blocks, buf.sel_count, None, buf.ws,
+                                                    stream)
+                    else:
+                        S.select(p, mode, t0, t1, None, buf, stream)
+                    S.scale_sparse_prefill_paged(p, mode, t0, t1, dev[0], kv, buf.unit_start, buf.n_units,
+                                                 buf.sel_blocks, buf.sel_count, buf.out, buf.ws, stream)
+                else:
+                    S.scale_build_reps_range(p, t0, t1, dev[0], dev[1], buf.reps, buf.fingerprints,
+                                             buf.unit_start, buf.n_units, buf.ws, stream)
+                    S.select(p, mode, t0, t1, dev[1], buf, stream)
+                    S.scale_sparse_prefill(p, mode, t0, t1, *dev, buf.unit_start, buf.n_units,
+                                           buf.sel_blocks, buf.sel_count, buf.out, buf.ws, stream)
+
+        for _ in range(2):
+            chunk_step()
+        torch.cuda.synchronize()
+        c_steps = max(3, args.steps // 2)
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for _ in range(c_steps):
+            chunk_step()
+        end.record(stream)
+        torch.cuda.synchronize()
+        st = S.scale_get_device_status(buf.ws)
+        if st != S.SCALE_OK:
+            raise RuntimeError(f"device status {st}: {S.status_string(st)}")
+        ms_c = start.elapsed_time(end) / c_steps
+        line["chunk_loop"] = {"ms_per_step": ms_c, "tokens_per_s": w.n_tokens / (ms_c / 1e3),
+                              "outer_chunks": len(chunks),
+                              "calls_per_step": 3 * len(chunks),
+                              "kernel_launches_per_step": launches(w, len(chunks), len(chunks))["total"],
+                              "loop": "per outer chunk: scale_build_reps_range, select, scale_sparse_prefill"}
+
     if not args.no_e2e:
         qh, kh, vh = (torch.from_numpy(x).pin_memory() for x in (q, k, v))
         oh = torch.empty(qh.shape, dtype=torch.int16).pin_memory()
@@ -656,9 +704,10 @@ def run_decode(args):
 def run_stack(args):
     """Multi-layer workload: attention-only TTFT of a chunked prefill over all layers.
 
-    Per step: scale_build_reps for every layer, then for each outer chunk (in
-    order) and each layer, scale_select and scale_sparse_prefill restricted to
-    that chunk's tokens -- the dependency order of a real chunked prefill."""
+    Per step, for each outer chunk (in order) and each layer: step (a) over the
+    chunk (scale_build_reps_range), then scale_select and scale_sparse_prefill
+    restricted to that chunk's tokens -- the dependency order of a real chunked
+    prefill, where a layer's Q, K and V of later chunks do not exist yet."""
     import torch
 
     world, rank, local = dist_setup(args)
@@ -687,11 +736,11 @@ def run_stack(args):
         n_attn = len(chunks) * len(layers)
 
         def step(ev=None):
-            for dev, b in zip(layers, bufs):
-                S.scale_build_reps(p, dev[0], dev[1], b.reps, b.fingerprints, b.unit_start, b.n_units, b.ws, stream)
             i = 0
             for t0, t1 in chunks:
                 for dev, b in zip(layers, bufs):
+                    S.scale_build_reps_range(p, t0, t1, dev[0], dev[1], b.reps, b.fingerprints, b.unit_start,
+                                             b.n_units, b.ws, stream)
                     S.select(p, mode, t0, t1, dev[1], b, stream)
                     if ev is not None:
                         ev[i][0].record(stream)
@@ -758,7 +807,7 @@ def run_stack(args):
                      "frac": achieved / peaks["bf16_sustained"], "frac_of_burst": achieved / peaks["bf16"],
                      "peak_source": f"bf16 sustained, of {peaks['source']}",
                      "algorithmic_flops_per_step": flops, "traffic": None},
-        "gpu_launches": args.steps * w.layers * launches(w, len(chunks))["total"],
+        "gpu_launches": args.steps * w.layers * launches(w, len(chunks), len(chunks))["total"],
         "clocks": clk,
     }
     if not args.no_baseline_mode and rank == 0:

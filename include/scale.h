@@ -150,8 +150,9 @@ int scale_build_reps_range(const scale_params_t *p, int64_t tok_begin, int64_t t
  * library holds until the process exits.
  *  - Limit: returns SCALE_ERR_WORKSPACE, without launching anything, when the
  *    scratch step (a) needs for `p` exceeds 16 MiB (it grows with
- *    M * ceil(L / 512) * H_q * 128 * 4 bytes; 4.2 MB for 128K tokens with
- *    L = 2048, 32 MB for 1M tokens with L = 4096, which is rejected).
+ *    M * (ceil(H_q / 2) + max_cluster_subchunks + 1) * 4 bytes plus 256; 34 KB
+ *    for 1M tokens with L = 4096, about 34 MB, which is rejected, for 128M
+ *    tokens with L = 512).
  *  - Set-up: the first call on each device looks up the array's device address
  *    with that device current; make that first call before any stream capture.
  *  - Sharing: every call on a device uses the same array, which keeps the last

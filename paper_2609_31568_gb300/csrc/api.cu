@@ -45,7 +45,7 @@ int derive(const scale_params_t* p, Derived* d)
     d->M = (d->N + d->L - 1) / d->L;
     d->nb = (d->N + d->B - 1) / d->B;
     d->D = d->Hq * kHeadDim;
-    d->fp_splits = (d->L + 511) / 512;
+    d->fp_groups = (d->D / 8 + 31) / 32;  // 32 sixteen-byte columns per fingerprint CTA
     d->theta = p->theta;
     d->sigma = p->select_scale;
     d->attn_scale = p->attn_scale > 0.f ? p->attn_scale : 1.0f / std::sqrt(static_cast<float>(kHeadDim));
@@ -62,8 +62,7 @@ WsLayout ws_layout(const Derived& d)
         return at;
     };
     w.status = take(256);
-    w.fp_partial = take(static_cast<size_t>(d.M) * d.fp_splits * d.D * sizeof(float));
-    w.norms = take(static_cast<size_t>(d.M) * sizeof(float));
+    w.fp_ss = take(static_cast<size_t>(d.M) * d.fp_groups * sizeof(float));
     w.gram = take(static_cast<size_t>(d.M) * d.S_max * sizeof(float));
     w.anchor = take(static_cast<size_t>(d.M) * sizeof(int32_t));
     const bool tok = d.B == 1;

@@ -5,8 +5,9 @@
 // plugin interface that hands over only the input and output buffers, or a
 // serving loop whose memory pool is fully reserved up front and where a
 // cudaMalloc (which may synchronise the device) is not allowed on the request
-// path. For them this entry point keeps step (a)'s scratch (fingerprint
-// partial sums, norms, the banded cosine matrix and the anchor flags) in the
+// path. For them this entry point keeps step (a)'s scratch (the sums of
+// squares of the fingerprints' column groups, the banded cosine matrix and
+// the anchor flags) in the
 // fixed array below, which every GPU that loads the library holds until the
 // process exits. The kernels and their launch are the ones of
 // scale_build_reps; only the scratch location differs.

@@ -3,7 +3,9 @@
 // anchor-based clustering (Eq. 8, Algorithm 1) inside each outer chunk.
 //
 // All four kernels stream their inputs once from HBM with 16-byte loads and
-// reduce in a fixed order, so their results are bit-reproducible run to run.
+// reduce in a fixed order, so their results are bit-reproducible run to run,
+// and each works on a range of outer chunks with the same per-element
+// arithmetic as over the whole sequence.
 #include <cuda_bf16.h>
 
 #include "scale_internal.h"
@@ -69,83 +71,87 @@ __global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k
     dst[1] = make_float4(acc[4] / cnt, acc[5] / cnt, acc[6] / cnt, acc[7] / cnt);
 }
 
-// Partial sums of the multi-head queries of sub-chunk i over token split s
-// (split_len tokens). Grid (sub-chunks [m0, m0 + gridDim.x), splits).
-__global__ void __launch_bounds__(512) k_fp_partial(const uint4* __restrict__ q, int64_t N, int D8,
-                                                     int L, int split_len, int splits, int64_t m0,
-                                                     float* __restrict__ partial)
+// Fingerprint v_i (Eq. 6): the mean of the multi-head queries of sub-chunk i.
+// One CTA per (sub-chunk, group of 32 sixteen-byte columns, i.e. 256 of the
+// H_q * 128 dimensions). Warp w sums the tokens w, w + 16, w + 32, ... of the
+// sub-chunk for its lane's column, so every token row is read as one 512-byte
+// span per warp; the 16 warps' sums are then added in warp order, divided by
+// |X_i| and written, together with the group's sum of squares (the norm of
+// Sec. V-A1 adds those in group order). The order is fixed, so the result is
+// bit-reproducible and the same for a sub-chunk whichever range of sub-chunks
+// a launch covers. Grid (sub-chunks [m0, m0 + gridDim.x), column groups).
+constexpr int kFpWarps = 16;
+constexpr int kFpGroupCols = 32;  // 16-byte columns per CTA
+
+__global__ void __launch_bounds__(32 * kFpWarps) k_fingerprint(const uint4* __restrict__ q, int64_t N, int D8,
+                                                               int L, int64_t m0, float* __restrict__ fp,
+                                                               float* __restrict__ ss_part)
 {
+    __shared__ float4 red[kFpWarps][kFpGroupCols * 2];
+    __shared__ float wsum[8];
     const int64_t i = m0 + blockIdx.x;
-    const int s = blockIdx.y;
-    const int64_t sc0 = i * L;
-    const int64_t sc1 = (sc0 + L < N) ? sc0 + L : N;
-    const int64_t t0 = sc0 + static_cast<int64_t>(s) * split_len;
-    const int64_t t1 = (t0 + split_len < sc1) ? t0 + split_len : sc1;
-    float* dst_row = partial + (i * splits + s) * static_cast<int64_t>(D8) * 8;
-    for (int c = threadIdx.x; c < D8; c += blockDim.x) {
-        float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    const int cg = blockIdx.y;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int c = cg * kFpGroupCols + lane;
+    const int64_t t0 = i * L;
+    const int64_t t1 = (t0 + L < N) ? t0 + L : N;
+    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    if (c < D8) {
         const uint4* src = q + c;
-        int64_t t = t0;
-        for (; t + 8 <= t1; t += 8) {
+        int64_t t = t0 + w;
+        for (; t + 7 * kFpWarps < t1; t += 8 * kFpWarps) {
             uint4 x[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) x[u] = ld_stream(src + (t + u) * D8);
+            for (int u = 0; u < 8; ++u) x[u] = ld_stream(src + (t + u * kFpWarps) * D8);
 #pragma unroll
             for (int u = 0; u < 8; ++u) add_bf16x8(acc, x[u]);
         }
-        for (; t < t1; ++t) add_bf16x8(acc, ld_stream(src + t * D8));
-        float4* dst = reinterpret_cast<float4*>(dst_row + c * 8);
-        dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
-        dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+        for (; t < t1; t += kFpWarps) add_bf16x8(acc, ld_stream(src + t * D8));
     }
-}
-
-// Deterministic block-wide sum (fixed shuffle tree, fixed warp order).
-__device__ float block_sum(float v, float* red)
-{
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) red[w] = v;
+    red[w][2 * lane] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    red[w][2 * lane + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
     __syncthreads();
-    float t = 0.f;
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < (blockDim.x + 31) / 32; ++i) t += red[i];
-        red[0] = t;
-    }
-    __syncthreads();
-    t = red[0];
-    __syncthreads();
-    return t;
-}
-
-// v_i = (sum of the partials in split order) / |X_i|, and ||v_i||_2, for
-// i in [m0, m0 + gridDim.x).
-__global__ void __launch_bounds__(512) k_fp_finalize(const float* __restrict__ partial, int D,
-                                                      int splits, int L, int64_t N, int64_t m0,
-                                                      float* __restrict__ fp,
-                                                      float* __restrict__ norms)
-{
-    __shared__ float red[32];
-    const int64_t i = m0 + blockIdx.x;
-    const int64_t cnt = ((i + 1) * L < N ? (i + 1) * L : N) - i * L;
-    const float inv_cnt = 1.0f / static_cast<float>(cnt);
-    float ss = 0.f;
-    for (int c = threadIdx.x; c < D; c += blockDim.x) {
+    if (threadIdx.x < kFpGroupCols * 8) {
+        // thread e owns element e of the group: column e / 8, lane e % 8 of it
+        const int e = threadIdx.x;
+        const float* flat = reinterpret_cast<const float*>(&red[0][0]);
         float v = 0.f;
-        for (int s = 0; s < splits; ++s) v += partial[(i * splits + s) * D + c];
-        v = v * inv_cnt;
-        fp[i * D + c] = v;
-        ss += v * v;
+        for (int ww = 0; ww < kFpWarps; ++ww) v += flat[ww * kFpGroupCols * 8 + e];
+        v = v / static_cast<float>(t1 - t0);
+        const int col = cg * kFpGroupCols + e / 8;
+        float sq = 0.f;
+        if (col < D8) {
+            fp[i * static_cast<int64_t>(D8) * 8 + static_cast<int64_t>(col) * 8 + (e & 7)] = v;
+            sq = v * v;
+        }
+        for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, o);
+        if (lane == 0) wsum[w] = sq;
     }
-    ss = block_sum(ss, red);
-    if (threadIdx.x == 0) norms[i] = sqrtf(ss);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float t = 0.f;
+        for (int ww = 0; ww < kFpGroupCols * 8 / 32; ++ww) t += wsum[ww];
+        ss_part[i * gridDim.y + cg] = t;
+    }
+}
+
+// ||v_i||_2 from the column groups' sums of squares, added in a fixed order
+// (lane-strided, then a butterfly that leaves the same value in every lane).
+// Warp-collective.
+__device__ __forceinline__ float fp_norm(const float* __restrict__ ss_part, int groups, int i)
+{
+    const int lane = threadIdx.x & 31;
+    float s = 0.f;
+    for (int g = lane; g < groups; g += 32) s += ss_part[static_cast<int64_t>(i) * groups + g];
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+    return sqrtf(s);
 }
 
 // gram[i][d] = cos(v_i, v_{i+d}) = v~_i . v~_{i+d} for 1 <= d < S_max and i+d
 // in the same outer chunk; 0 when either norm is 0. One warp per (i, d);
 // one CTA per i in [m0, m0 + gridDim.x).
-__global__ void k_gram(const float* __restrict__ fp, const float* __restrict__ norms, int D, int M,
-                       int S_max, int per_outer, int m0, float* __restrict__ gram)
+__global__ void k_gram(const float* __restrict__ fp, const float* __restrict__ ss_part, int groups, int D,
+                       int M, int S_max, int per_outer, int m0, float* __restrict__ gram)
 {
     const int i = m0 + static_cast<int>(blockIdx.x);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -159,10 +165,8 @@ __global__ void k_gram(const float* __restrict__ fp, const float* __restrict__ n
         float s = 0.f;
         for (int c = lane; c < D; c += 32) s = fmaf(a[c], b[c], s);
         for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-        if (lane == 0) {
-            const float na = norms[i], nb = norms[j];
-            gram[static_cast<int64_t>(i) * S_max + d] = (na > 0.f && nb > 0.f) ? s / (na * nb) : 0.f;
-        }
+        const float na = fp_norm(ss_part, groups, i), nb = fp_norm(ss_part, groups, j);  // whole warp
+        if (lane == 0) gram[static_cast<int64_t>(i) * S_max + d] = (na > 0.f && nb > 0.f) ? s / (na * nb) : 0.f;
     }
 }
 
@@ -254,8 +258,7 @@ cudaError_t launch_build_reps_range(const Derived& d, const void* q, const void*
 {
     if (c_begin < 0 || c_end > outer_chunks(d) || c_begin >= c_end) return cudaSuccess;
     const WsLayout lay = ws_layout(d);
-    float* partial = reinterpret_cast<float*>(ws + lay.fp_partial);
-    float* norms = reinterpret_cast<float*>(ws + lay.norms);
+    float* ss_part = reinterpret_cast<float*>(ws + lay.fp_ss);
     float* gram = reinterpret_cast<float*>(ws + lay.gram);
     int32_t* flag = reinterpret_cast<int32_t*>(ws + lay.anchor);
 
@@ -277,15 +280,13 @@ cudaError_t launch_build_reps_range(const Derived& d, const void* q, const void*
             static_cast<const uint4*>(k), pg, d.N, row_chunks, d.B, d.nb, b0, reps);
 
     const int D8 = d.D / 8;
-    const int split_len = (d.L + d.fp_splits - 1) / d.fp_splits;
     const unsigned nm = static_cast<unsigned>(m1 - m0);
-    k_fp_partial<<<dim3(nm, d.fp_splits), D8 < 512 ? D8 : 512, 0, st>>>(
-        static_cast<const uint4*>(q), d.N, D8, d.L, split_len, d.fp_splits, m0, partial);
-    k_fp_finalize<<<nm, 512, 0, st>>>(partial, d.D, d.fp_splits, d.L, d.N, m0, fingerprints, norms);
+    k_fingerprint<<<dim3(nm, d.fp_groups), 32 * kFpWarps, 0, st>>>(static_cast<const uint4*>(q), d.N, D8, d.L,
+                                                                   m0, fingerprints, ss_part);
     if (d.S_max > 1) {
         const int warps = d.S_max - 1 < 16 ? d.S_max - 1 : 16;
-        k_gram<<<nm, 32 * warps, 0, st>>>(fingerprints, norms, d.D, static_cast<int>(d.M), d.S_max,
-                                          d.per_outer, static_cast<int>(m0), gram);
+        k_gram<<<nm, 32 * warps, 0, st>>>(fingerprints, ss_part, d.fp_groups, d.D, static_cast<int>(d.M),
+                                          d.S_max, d.per_outer, static_cast<int>(m0), gram);
     }
     k_cluster<<<1, 1024, 0, st>>>(gram, static_cast<int>(d.M), d.S_max, d.per_outer, d.theta, c_begin,
                                   c_end, flag, unit_start, n_units);

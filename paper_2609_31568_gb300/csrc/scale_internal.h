@@ -32,15 +32,14 @@ struct Derived {
     int64_t M;       // sub-chunks
     int64_t nb;      // blocks
     int D;           // H_q * d_h
-    int fp_splits;   // token splits of the fingerprint reduction
+    int fp_groups;   // 256-dimension column groups of the fingerprint reduction
     float theta, sigma, attn_scale;
 };
 
 // Workspace regions (byte offsets from the workspace base).
 struct WsLayout {
     size_t status;      // int32 status word (+ padding)
-    size_t fp_partial;  // fp32 [M][fp_splits][D]
-    size_t norms;       // fp32 [M]
+    size_t fp_ss;       // fp32 [M][fp_groups]: sums of squares of the fingerprint's column groups
     size_t gram;        // fp32 [M][S_max]   cosine of sub-chunk i with i+d
     size_t anchor;      // int32 [M]         1 if sub-chunk i opens a cluster
     size_t logits;      // fp32 [M][H_q][nb]     (block size > 1 only)

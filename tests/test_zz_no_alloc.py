@@ -67,7 +67,9 @@ def test_noalloc_build_reps_matches_workspace_entry_point_twice():
 def test_noalloc_refuses_problems_beyond_its_scratch():
     pkg.build()
     S.load()
-    p = S.params_for(workload("llama8b-1m"))  # needs 32 MiB of step (a) scratch
+    # 128M tokens in 512-token sub-chunks: M = 262144 sub-chunks, whose norm
+    # sums and banded cosine rows need about 34 MB of step (a) scratch
+    p = S.params_for(workload("llama8b-1m"), n_tokens=1 << 27, sub_chunk=512)
     small = torch.zeros(1024, dtype=torch.float32, device="cuda")
     ints = torch.zeros(1024, dtype=torch.int32, device="cuda")
     with pytest.raises(S.ScaleError) as e:
