@@ -32,7 +32,7 @@ from synth import generate_layer, workload  # noqa: E402
 METRIC = "sparse-prefill tokens/sec and TTFT at 128K ctx on 1 GB300; % of roofline"
 DEFAULT_WORKLOAD = "llama8b-128k"
 KERNEL_SRC = os.path.join(ROOT, "paper_2609_31568_gb300", "csrc", "attn.cu")
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "attn_llama8b-128k_ncu.md")
+PROFILE_DIR = os.path.join(ROOT, "profiles")
 
 
 def parse_args():
@@ -80,7 +80,7 @@ def launches(w, selects: int = 1, builds: int = 1) -> dict:
     scores in four kernels and gathers the distant keys through a per-unit
     list)."""
     tok = w.block_size == 1
-    build = (3 if tok else 4) + (1 if w.max_cluster_subchunks > 1 else 0)
+    build = (2 if tok else 3) + (1 if w.max_cluster_subchunks > 1 else 0)
     # the top-k is one kernel, or 12 (init, 4 x (histogram, pick), count, scan,
     # emit) for units of more than 64K candidates
     topk = 12 if tok and w.n_blocks > 65536 else 1
@@ -88,6 +88,26 @@ def launches(w, selects: int = 1, builds: int = 1) -> dict:
     attend = 3 if tok else 1
     return {"build_reps": build * builds, "select": select * selects, "attend": attend * selects,
             "total": build * builds + (select + attend) * selects}
+
+
+def host_link_gbs(host, dev_bytes, stream) -> dict:
+    """H2D and D2H bandwidth of one pinned copy each way (up to 512 MB), timed
+    with CUDA events: what the host link gave the end-to-end call on this machine."""
+    import torch
+
+    n = min(host.numel() * host.element_size(), dev_bytes.numel(), 512 << 20)
+    src = host.view(torch.uint8).reshape(-1)[:n]
+    dst = dev_bytes[:n]
+    out = {}
+    for name, (a, b) in (("h2d", (dst, src)), ("d2h", (src, dst))):
+        a.copy_(b, non_blocking=True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        a.copy_(b, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        out[name] = n / (e0.elapsed_time(e1) / 1e3) / 1e9
+    return out
 
 
 def key_counts(w, unit_start, n_units, sel, cnt, per_subchunk):
@@ -108,15 +128,17 @@ def key_counts(w, unit_start, n_units, sel, cnt, per_subchunk):
     return total
 
 
-def profile_traffic():
-    """Per-launch DRAM bytes of the attention kernel from the committed ncu
-    summary, or None when the kernel source changed since the capture."""
-    if not os.path.exists(PROFILE_SUMMARY):
+def profile_traffic(workload_name: str):
+    """Per-launch DRAM bytes of the attention kernel on this workload from the
+    committed ncu summary (profiles/attn_<workload>_ncu.md), or None when there
+    is none or the kernel source changed since the capture."""
+    summary = os.path.join(PROFILE_DIR, f"attn_{workload_name}_ncu.md")
+    if not os.path.exists(summary):
         return None
     with open(KERNEL_SRC, "rb") as f:
         sha = hashlib.sha256(f.read()).hexdigest()[:16]
     vals = {}
-    with open(PROFILE_SUMMARY) as f:
+    with open(summary) as f:
         for line in f:
             if ": " in line and line.strip().startswith("- "):
                 k, v = line.strip()[2:].split(": ", 1)  # keys may hold a colon ("sha256[:16]")
@@ -400,7 +422,7 @@ def run_scale(args):
                      "frac": achieved / peaks["bf16_sustained"],
                      "frac_of_burst": achieved / peaks["bf16"],
                      "peak_source": f"bf16 sustained, of {peaks['source']}",
-                     "algorithmic_flops_per_launch": flops, "traffic": profile_traffic()},
+                     "algorithmic_flops_per_launch": flops, "traffic": profile_traffic(w.name)},
         "gpu_launches": args.steps * launches(w)["total"],
         "clocks": clk,
     }
@@ -470,12 +492,15 @@ def run_scale(args):
         arena = torch.empty(S.scale_prefill_host_arena_size(p, mode), dtype=torch.uint8, device="cuda")
         S.scale_prefill_host(p, mode, qh, kh, vh, oh, arena, stream)
         reps = max(3, args.steps // 4)
+        link = host_link_gbs(qh, arena, stream)
         torch.cuda.synchronize()
         barrier()
-        t0 = time.perf_counter()
+        per_call = []
         for _ in range(reps):
+            t0 = time.perf_counter()
             S.scale_prefill_host(p, mode, qh, kh, vh, oh, arena, stream)
-        t_e2e = (time.perf_counter() - t0) / reps
+            per_call.append(time.perf_counter() - t0)
+        t_e2e = sum(per_call) / reps
         if world > 1:
             t = torch.tensor([t_e2e], device="cuda")
             torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
@@ -483,6 +508,8 @@ def run_scale(args):
         line["e2e"] = {"value": world * w.n_tokens / t_e2e, "unit": "tokens/s",
                        "h2d_bytes_per_step": int(q.nbytes + k.nbytes + v.nbytes),
                        "d2h_bytes_per_step": int(q.nbytes), "ms_per_step": t_e2e * 1e3,
+                       "ms_min": min(per_call) * 1e3, "ms_median": statistics.median(per_call) * 1e3,
+                       "host_link_gbs": link,
                        "api": "scale_prefill_host (pinned host buffers)"}
         del arena
 
