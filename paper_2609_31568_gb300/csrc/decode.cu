@@ -16,8 +16,8 @@
 //  - attention (Eq. 10 for one row): keys = sinks U selection U [W_t, t].
 //
 // Scoring one query against every key is a matrix-vector product: it runs on
-// the CUDA cores, one warp per key, reading K once with 8-byte loads per lane
-// (the step is bound by HBM, not by arithmetic). Whether the step retrieves is
+// the CUDA cores, one thread per key, reading K once in 16-byte pieces (the
+// step is bound by HBM, not by arithmetic). Whether the step retrieves is
 // decided on the device, so a step never synchronises with the host.
 #include <cuda_bf16.h>
 
@@ -34,8 +34,20 @@ constexpr size_t kDecUnits = 64;    // int32[2] unit table [t, t + 1] of the anc
 constexpr size_t kDecAnchor = 256;  // fp32 [H_q * 128]
 // selection int32 [k] and its count follow the anchor
 
+// Read-only 16-byte load; volatile keeps a run of them issued back to back.
+__device__ __forceinline__ uint4 ld_nc(const uint4* p)
+{
+    uint4 r;
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+    return r;
+}
+
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+constexpr int kDecSplits = 128;
 
 struct DecArgs {
     int Hq, Hkv, g;
@@ -53,8 +65,8 @@ struct DecArgs {
     float* scores;      // [cap]
     float* part;        // [H_q][splits][130]: max, sum, o[128]
     int splits;
-    float2* zpart;      // [chunks][H_q] (max, sum) of each candidate chunk
-    int chunk;          // candidates per logits CTA
+    float2* zpart;      // [H_q][n_stat] (max, sum) of each 64-candidate chunk
+    int n_stat;         // 64-candidate chunks of the candidates
 };
 
 __host__ __device__ __forceinline__ int64_t window_start(const DecArgs& a, int64_t t)
@@ -117,80 +129,212 @@ __global__ void __launch_bounds__(256) k_dec_gate(DecArgs a, const __nv_bfloat16
         for (int i = threadIdx.x; i < D; i += blockDim.x) a.anchor[i] = __bfloat162float(q[i]);
 }
 
-// z[h][c] = sigma * q^(h) . k_c^(h / g) for the candidates c of this CTA's
-// chunk [lo + chunk * blockIdx.x, + chunk): one thread per key, streaming its
-// K row in 16-byte pieces (the query, in shared memory, is read as
-// broadcasts). The chunk's logits are staged in shared memory, written out as
-// whole rows, and summarised per head as (max, sum of exp(z - max)).
-__global__ void __launch_bounds__(128) k_dec_logits(DecArgs a, const __nv_bfloat16* __restrict__ q,
+// Merge of two (max, sum of exp(z - max)) summaries; symmetric in its
+// arguments, so both lanes of a butterfly get the same bits.
+__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2)
+{
+    const float mn = fmaxf(m, m2);
+    s = (m == -INFINITY ? 0.f : s * expf(m - mn)) + (m2 == -INFINITY ? 0.f : s2 * expf(m2 - mn));
+    m = mn;
+}
+
+// z[h][c] = sigma * q^(h) . k_c^(h / g) for the candidates c in
+// [n_sink, W_t), G = g query heads per KV head. A CTA takes 512 candidates,
+// warp w the 64 from c0 + 64 w: lane l the four keys c0 + 64 w + l / 2 + 16 r
+// (r < 4) and the 16-byte pieces l % 2, l % 2 + 2, ... of each key's 256-byte
+// row for KV head j, so each load instruction reads 16 keys x one whole
+// 32-byte sector. A query piece read from shared memory feeds the four keys
+// (shared-memory traffic per key is a quarter of one key per thread), every
+// key piece is unpacked once for the G heads, one shuffle joins the halves.
+// Each warp writes its logits straight to z and summarises every head over
+// its 64 keys as (max, sum of exp(z - max)) in zpart[h][chunk], chunk =
+// 8 blockIdx.x + w, merged across lanes by a fixed butterfly.
+constexpr int kDecStat = 64;         // candidates per (max, sum) summary
+constexpr int kDecBlockKeys = 512;   // candidates per CTA of k_dec_logits
+
+template <int G>
+__global__ void __launch_bounds__(256) k_dec_logits(DecArgs a, const __nv_bfloat16* __restrict__ q,
                                                     const uint4* __restrict__ k)
 {
     if (!a.state[2]) return;
-    extern __shared__ float sm[];
-    float* qs = sm;                        // [H_q][128]
-    float* zs = sm + a.Hq * kHeadDim;      // [H_q][chunk]
+    extern __shared__ float qs[];  // [H_q][128]
     const int D = a.Hq * kHeadDim;
     for (int i = threadIdx.x; i < D; i += blockDim.x) qs[i] = __bfloat162float(q[i]);
     __syncthreads();
     const int64_t lo = a.n_sink, hi = window_start(a, a.t);
-    const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * a.chunk;
-    const int n = static_cast<int>((hi - c0 < a.chunk) ? hi - c0 : a.chunk);
-    const int i = threadIdx.x;
-    if (i < n) {
-        const int64_t c = c0 + i;
-        for (int j = 0; j < a.Hkv; ++j) {
-            const uint4* kr = k + (c * a.Hkv + j) * 16;  // 16 pieces of 8 bf16
-            uint4 kv[16];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, half = lane & 1;
+    const int64_t cw = lo + static_cast<int64_t>(blockIdx.x) * kDecBlockKeys + kDecStat * warp;
+    if (cw >= hi) return;  // warp-uniform; no barrier follows
+    const int64_t cl = cw + (lane >> 1);
+    const int64_t chunk = static_cast<int64_t>(blockIdx.x) * (kDecBlockKeys / kDecStat) + warp;
+    bool live[4];
 #pragma unroll
-            for (int p = 0; p < 16; ++p) kv[p] = kr[p];
-            for (int hl = 0; hl < a.g; ++hl) {
-                const float4* qh = reinterpret_cast<const float4*>(qs + (j * a.g + hl) * kHeadDim);
-                float acc = 0.f;
+    for (int r = 0; r < 4; ++r) live[r] = cl + 16 * r < hi;
+    const uint4 zero = make_uint4(0, 0, 0, 0);
+    constexpr int UU = G <= 4 ? 2 : 1;  // pieces per key in flight together (registers)
+    for (int j = 0; j < a.Hkv; ++j) {
+        float acc[4][G];
 #pragma unroll
-                for (int p = 0; p < 16; ++p) {
-                    const float4 qa = qh[2 * p], qb = qh[2 * p + 1];
-                    acc += qa.x * bf16_lo(kv[p].x) + qa.y * bf16_hi(kv[p].x) + qa.z * bf16_lo(kv[p].y) +
-                           qa.w * bf16_hi(kv[p].y) + qb.x * bf16_lo(kv[p].z) + qb.y * bf16_hi(kv[p].z) +
-                           qb.z * bf16_lo(kv[p].w) + qb.w * bf16_hi(kv[p].w);
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+            for (int hl = 0; hl < G; ++hl) acc[r][hl] = 0.f;
+        const uint4* kr = k + (cl * a.Hkv + j) * 16 + half;
+        const int64_t key_step = static_cast<int64_t>(16) * a.Hkv * 16;  // 16 keys, in uint4
+        const float* qj = qs + j * G * kHeadDim + 8 * half;
+#pragma unroll
+        for (int u0 = 0; u0 < 8; u0 += UU) {
+            uint4 kv[UU][4];
+#pragma unroll
+            for (int uu = 0; uu < UU; ++uu)
+#pragma unroll
+                for (int r = 0; r < 4; ++r)
+                    kv[uu][r] = live[r] ? ld_nc(kr + r * key_step + 2 * (u0 + uu)) : zero;
+#pragma unroll
+            for (int uu = 0; uu < UU; ++uu) {
+                float4 qa[G], qb[G];
+#pragma unroll
+                for (int hl = 0; hl < G; ++hl) {
+                    const float4* qh = reinterpret_cast<const float4*>(qj + hl * kHeadDim + 16 * (u0 + uu));
+                    qa[hl] = qh[0];
+                    qb[hl] = qh[1];
                 }
-                zs[(j * a.g + hl) * a.chunk + i] = a.sigma * acc;
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    const uint4 w = kv[uu][r];
+                    const float x0 = bf16_lo(w.x), x1 = bf16_hi(w.x), x2 = bf16_lo(w.y), x3 = bf16_hi(w.y);
+                    const float x4 = bf16_lo(w.z), x5 = bf16_hi(w.z), x6 = bf16_lo(w.w), x7 = bf16_hi(w.w);
+#pragma unroll
+                    for (int hl = 0; hl < G; ++hl)
+                        acc[r][hl] += qa[hl].x * x0 + qa[hl].y * x1 + qa[hl].z * x2 + qa[hl].w * x3 +
+                                      qb[hl].x * x4 + qb[hl].y * x5 + qb[hl].z * x6 + qb[hl].w * x7;
+                }
             }
+        }
+#pragma unroll
+        for (int hl = 0; hl < G; ++hl) {
+            const int h = j * G + hl;
+            float zv[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) zv[r] = a.sigma * (acc[r][hl] + __shfl_xor_sync(0xFFFFFFFFu, acc[r][hl], 1));
+            float* zh = a.z + static_cast<int64_t>(h) * a.cap;
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+                if ((r >> 1) == half && live[r]) zh[cl + 16 * r] = zv[r];  // half 0: keys 0, 1; half 1: 2, 3
+            float m = -INFINITY;
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+                if (live[r]) m = fmaxf(m, zv[r]);
+            float sum = 0.f;
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+                if (live[r]) sum += expf(zv[r] - m);
+            for (int o = 2; o < 32; o <<= 1)  // the two lanes of a key hold the same values
+                merge_ms(m, sum, __shfl_xor_sync(0xFFFFFFFFu, m, o), __shfl_xor_sync(0xFFFFFFFFu, sum, o));
+            if (lane == 0) a.zpart[static_cast<int64_t>(h) * a.n_stat + chunk] = make_float2(m, sum);
+        }
+    }
+}
+
+// Any group size: two lanes per key (every other 16-byte piece of its row),
+// the query heads of the KV head looped at run time; 128 candidates per CTA,
+// logits staged in shared memory and summarised per 64 keys as above.
+__global__ void __launch_bounds__(256) k_dec_logits_any(DecArgs a, const __nv_bfloat16* __restrict__ q,
+                                                        const uint4* __restrict__ k)
+{
+    if (!a.state[2]) return;
+    extern __shared__ float sm[];
+    float* qs = sm;                        // [H_q][128]
+    float* zs = sm + a.Hq * kHeadDim;      // [H_q][128]
+    const int D = a.Hq * kHeadDim;
+    for (int i = threadIdx.x; i < D; i += blockDim.x) qs[i] = __bfloat162float(q[i]);
+    __syncthreads();
+    const int64_t lo = a.n_sink, hi = window_start(a, a.t);
+    const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * 128;
+    const int n = static_cast<int>((hi - c0 < 128) ? hi - c0 : 128);
+    const int i = threadIdx.x >> 1, half = threadIdx.x & 1;
+    const bool live = i < n;
+    const uint4 zero = make_uint4(0, 0, 0, 0);
+    for (int j = 0; j < a.Hkv; ++j) {
+        const uint4* kr = k + ((c0 + i) * a.Hkv + j) * 16 + half;
+        uint4 kv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) kv[u] = live ? ld_nc(kr + 2 * u) : zero;
+        for (int hl = 0; hl < a.g; ++hl) {
+            const float4* qh = reinterpret_cast<const float4*>(qs + (j * a.g + hl) * kHeadDim + 8 * half);
+            float acc = 0.f;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const float4 qa = qh[4 * u], qb = qh[4 * u + 1];
+                acc += qa.x * bf16_lo(kv[u].x) + qa.y * bf16_hi(kv[u].x) + qa.z * bf16_lo(kv[u].y) +
+                       qa.w * bf16_hi(kv[u].y) + qb.x * bf16_lo(kv[u].z) + qb.y * bf16_hi(kv[u].z) +
+                       qb.z * bf16_lo(kv[u].w) + qb.w * bf16_hi(kv[u].w);
+            }
+            acc += __shfl_xor_sync(0xFFFFFFFFu, acc, 1);
+            if (live && !half) zs[(j * a.g + hl) * 128 + i] = a.sigma * acc;
         }
     }
     __syncthreads();
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int h = warp; h < a.Hq; h += blockDim.x / 32) {
-        const float* zh = zs + h * a.chunk;
-        float* dst = a.z + h * a.cap + c0;
+    for (int hs = warp; hs < 2 * a.Hq; hs += blockDim.x / 32) {
+        const int h = hs >> 1, sub = hs & 1;
+        const int b0 = sub * kDecStat, b1 = n < b0 + kDecStat ? n : b0 + kDecStat;
+        if (b1 <= b0) continue;  // past the candidates: never read
+        const float* zh = zs + h * 128;
+        float* dst = a.z + static_cast<int64_t>(h) * a.cap + c0;
         float m = -INFINITY;
-        for (int ii = lane; ii < n; ii += 32) {
+        for (int ii = b0 + lane; ii < b1; ii += 32) {
             dst[ii] = zh[ii];
             m = fmaxf(m, zh[ii]);
         }
         for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
         float sum = 0.f;
-        for (int ii = lane; ii < n; ii += 32) sum += expf(zh[ii] - m);
+        for (int ii = b0 + lane; ii < b1; ii += 32) sum += expf(zh[ii] - m);
         for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
-        if (lane == 0) a.zpart[static_cast<int64_t>(blockIdx.x) * a.Hq + h] = make_float2(m, sum);
+        if (lane == 0) a.zpart[static_cast<int64_t>(h) * a.n_stat + blockIdx.x * 2 + sub] = make_float2(m, sum);
     }
 }
 
-// Per head (one warp): the chunks' (max, sum) merged into max and 1 / sum.
+// Fixed-order block reductions (warp butterflies, then the warps in order).
+__device__ __forceinline__ float block_max256(float v, float* red)
+{
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float m = red[0];
+    for (int w = 1; w < static_cast<int>(blockDim.x >> 5); ++w) m = fmaxf(m, red[w]);
+    __syncthreads();
+    return m;
+}
+
+__device__ __forceinline__ float block_sum256(float v, float* red)
+{
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+    __syncthreads();
+    float s = red[0];
+    for (int w = 1; w < static_cast<int>(blockDim.x >> 5); ++w) s += red[w];
+    __syncthreads();
+    return s;
+}
+
+// Per head (one CTA of 256 threads): the chunks' (max, sum) merged into max
+// and 1 / sum, thread t taking the chunks t, t + 256, ... in order.
 __global__ void __launch_bounds__(256) k_dec_stats(DecArgs a, int n_chunks)
 {
     if (!a.state[2]) return;
-    const int h = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-    if (h >= a.Hq) return;
+    __shared__ float red[8];
+    const int h = blockIdx.x;
+    const float2* zp = a.zpart + static_cast<int64_t>(h) * n_chunks;
     float m = -INFINITY;
-    for (int b = lane; b < n_chunks; b += 32) m = fmaxf(m, a.zpart[static_cast<int64_t>(b) * a.Hq + h].x);
-    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+    for (int b = threadIdx.x; b < n_chunks; b += blockDim.x) m = fmaxf(m, zp[b].x);
+    m = block_max256(m, red);
     float s = 0.f;
-    for (int b = lane; b < n_chunks; b += 32) {
-        const float2 p = a.zpart[static_cast<int64_t>(b) * a.Hq + h];
+    for (int b = threadIdx.x; b < n_chunks; b += blockDim.x) {
+        const float2 p = zp[b];
         if (p.x > -INFINITY) s += p.y * expf(p.x - m);
     }
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-    if (lane == 0) a.stats[h] = make_float2(m, s > 0.f ? 1.0f / s : 0.f);
+    s = block_sum256(s, red);
+    if (threadIdx.x == 0) a.stats[h] = make_float2(m, s > 0.f ? 1.0f / s : 0.f);
 }
 
 // score[c] = sum over heads (in order) of exp(z - max) / sum; NaN off the candidates.
@@ -216,7 +360,9 @@ __global__ void __launch_bounds__(256) k_dec_vote(DecArgs a)
 // cached selection (produced by the top-k: ascending, inside [n_sink, W_a)
 // with W_a <= W_t), then the window [W_t, t]. One warp per query head of KV
 // head blockIdx.x, lane l holding dimensions [4 l, 4 l + 4); online softmax in
-// log2 units. Writes (max, sum, unnormalised o) per (head, split).
+// log2 units, four keys per update (their loads and dot products are
+// independent, so they overlap). Writes (max, sum, unnormalised o) per
+// (head, split).
 __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16* __restrict__ q,
                                                   const uint2* __restrict__ k, const uint2* __restrict__ v)
 {
@@ -235,10 +381,49 @@ __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16
     const float q0 = __bfloat162float(qh[0]), q1 = __bfloat162float(qh[1]);
     const float q2 = __bfloat162float(qh[2]), q3 = __bfloat162float(qh[3]);
     float m = -INFINITY, l = 0.f, o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
-#pragma unroll 4
-    for (int i = i0; i < i1; ++i) {
-        const int64_t tok = i < n_s ? i : (i < n_s + n_sel ? a.sel[i - n_s] : W + (i - n_s - n_sel));
-        const int64_t row = (tok * a.Hkv + j) * 32 + lane;
+    auto key = [&](int i) -> int64_t {
+        return i < n_s ? i : (i < n_s + n_sel ? a.sel[i - n_s] : W + (i - n_s - n_sel));
+    };
+    int i = i0;
+    for (; i + 4 <= i1; i += 4) {
+        uint2 kw[4], vw[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t row = (key(i + u) * a.Hkv + j) * 32 + lane;
+            kw[u] = k[row];
+            vw[u] = v[row];
+        }
+        float s[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            s[u] = q0 * bf16_lo(kw[u].x) + q1 * bf16_hi(kw[u].x) + q2 * bf16_lo(kw[u].y) + q3 * bf16_hi(kw[u].y);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int u = 0; u < 4; ++u) s[u] += __shfl_xor_sync(0xFFFFFFFFu, s[u], o);
+        float m_new = m;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            s[u] *= a.attn_scale_log2;
+            m_new = fmaxf(m_new, s[u]);
+        }
+        const float alpha = exp2f(m - m_new);
+        float p[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) p[u] = exp2f(s[u] - m_new);
+        l = l * alpha + (((p[0] + p[1]) + p[2]) + p[3]);
+        o0 = o0 * alpha + p[0] * bf16_lo(vw[0].x) + p[1] * bf16_lo(vw[1].x) + p[2] * bf16_lo(vw[2].x) +
+             p[3] * bf16_lo(vw[3].x);
+        o1 = o1 * alpha + p[0] * bf16_hi(vw[0].x) + p[1] * bf16_hi(vw[1].x) + p[2] * bf16_hi(vw[2].x) +
+             p[3] * bf16_hi(vw[3].x);
+        o2 = o2 * alpha + p[0] * bf16_lo(vw[0].y) + p[1] * bf16_lo(vw[1].y) + p[2] * bf16_lo(vw[2].y) +
+             p[3] * bf16_lo(vw[3].y);
+        o3 = o3 * alpha + p[0] * bf16_hi(vw[0].y) + p[1] * bf16_hi(vw[1].y) + p[2] * bf16_hi(vw[2].y) +
+             p[3] * bf16_hi(vw[3].y);
+        m = m_new;
+    }
+    for (; i < i1; ++i) {
+        const int64_t row = (key(i) * a.Hkv + j) * 32 + lane;
         const uint2 kw = k[row];
         const uint2 vw = v[row];
         float s = q0 * bf16_lo(kw.x) + q1 * bf16_hi(kw.x) + q2 * bf16_lo(kw.y) + q3 * bf16_hi(kw.y);
@@ -265,20 +450,27 @@ __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16
 }
 
 // Merge the splits of every head (in order) and write the bf16 output row.
+// One CTA per head: thread s weighs split s (2^(m_s - m)), then thread d adds
+// the weighted split outputs of dimension d in split order.
 __global__ void __launch_bounds__(128) k_dec_combine(DecArgs a, __nv_bfloat16* __restrict__ out)
 {
+    __shared__ float w_s[kDecSplits];
+    __shared__ float red[4];
     const int h = blockIdx.x, d = threadIdx.x;
     const float* ph = a.part + static_cast<int64_t>(h) * a.splits * 130;
     float m = -INFINITY;
-    for (int s = 0; s < a.splits; ++s) m = fmaxf(m, ph[s * 130]);
-    float l = 0.f, o = 0.f;
-    for (int s = 0; s < a.splits; ++s) {
+    for (int s = threadIdx.x; s < a.splits; s += blockDim.x) m = fmaxf(m, ph[s * 130]);
+    m = block_max256(m, red);
+    float l = 0.f;
+    for (int s = threadIdx.x; s < a.splits; s += blockDim.x) {
         const float ms = ph[s * 130];
-        if (ms == -INFINITY) continue;
-        const float w = exp2f(ms - m);
+        const float w = ms == -INFINITY ? 0.f : exp2f(ms - m);
+        w_s[s] = w;
         l += ph[s * 130 + 1] * w;
-        o += ph[s * 130 + 2 + d] * w;
     }
+    l = block_sum256(l, red);  // its barriers also publish w_s
+    float o = 0.f;
+    for (int s = 0; s < a.splits; ++s) o += ph[s * 130 + 2 + d] * w_s[s];
     out[h * kHeadDim + d] = __float2bfloat16_rn(l > 0.f ? o / l : 0.f);
 }
 
@@ -299,13 +491,12 @@ size_t decode_ws_bytes(const Derived& d, int splits)
     off = align_up(off + static_cast<size_t>(d.Hq) * sizeof(float2), kAlign);   // stats
     off = align_up(off + cap * sizeof(float), kAlign);                          // scores
     off = align_up(off + static_cast<size_t>(d.Hq) * splits * 130 * sizeof(float), kAlign);
-    off = align_up(off + static_cast<size_t>(d.Hq) * ((cap + 127) / 128) * sizeof(float2), kAlign);  // zpart
+    off = align_up(off + static_cast<size_t>(d.Hq) * ((cap + kDecStat - 1) / kDecStat) * sizeof(float2), kAlign);  // zpart
     off = align_up(off + (256 + 4) * sizeof(int32_t), kAlign);                                    // top-k hist, state
     off = align_up(off + static_cast<size_t>(topk_max_chunks(d)) * sizeof(int2), kAlign);          // top-k counts
     return off;
 }
 
-constexpr int kDecSplits = 128;
 
 int decode_splits() { return kDecSplits; }
 
@@ -342,8 +533,8 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
     a.stats = reinterpret_cast<float2*>(ws + take(static_cast<size_t>(d.Hq) * sizeof(float2)));
     a.scores = reinterpret_cast<float*>(ws + take(cap * sizeof(float)));
     a.part = reinterpret_cast<float*>(ws + take(static_cast<size_t>(d.Hq) * kDecSplits * 130 * sizeof(float)));
-    a.zpart = reinterpret_cast<float2*>(ws + take(static_cast<size_t>(d.Hq) * ((cap + 127) / 128) * sizeof(float2)));
-    a.chunk = 128;  // 32 KB of staged logits for 32 heads: several CTAs per SM keep loads in flight
+    a.zpart = reinterpret_cast<float2*>(
+        ws + take(static_cast<size_t>(d.Hq) * ((cap + kDecStat - 1) / kDecStat) * sizeof(float2)));
     int32_t* tk_hist = reinterpret_cast<int32_t*>(ws + take((256 + 4) * sizeof(int32_t)));
     int2* tk_counts = reinterpret_cast<int2*>(ws + take(static_cast<size_t>(topk_max_chunks(d)) * sizeof(int2)));
 
@@ -351,13 +542,25 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
     k_dec_gate<<<1, 256, 0, st>>>(a, qb);
     const int64_t n_cand = window_start(a, t) - d.n_sink;
     if (n_cand > 0) {
-        const int n_chunks = static_cast<int>((n_cand + a.chunk - 1) / a.chunk);
-        const size_t smem = (static_cast<size_t>(d.Hq) * kHeadDim + static_cast<size_t>(d.Hq) * a.chunk) * sizeof(float);
-        cudaError_t e0 = cudaFuncSetAttribute(k_dec_logits, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              static_cast<int>(smem));
-        if (e0 != cudaSuccess) return e0;
-        k_dec_logits<<<n_chunks, 128, smem, st>>>(a, qb, static_cast<const uint4*>(k));
-        k_dec_stats<<<(d.Hq + 7) / 8, 256, 0, st>>>(a, n_chunks);
+        a.n_stat = static_cast<int>((n_cand + kDecStat - 1) / kDecStat);
+        cudaError_t e0;
+        if (d.g == 1 || d.g == 2 || d.g == 4 || d.g == 8) {
+            auto kern = d.g == 1 ? k_dec_logits<1> : d.g == 2 ? k_dec_logits<2> : d.g == 4 ? k_dec_logits<4>
+                                                                                         : k_dec_logits<8>;
+            const size_t smem = static_cast<size_t>(d.Hq) * kHeadDim * sizeof(float);
+            e0 = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            if (e0 != cudaSuccess) return e0;
+            kern<<<static_cast<unsigned>((n_cand + kDecBlockKeys - 1) / kDecBlockKeys), 256, smem, st>>>(
+                a, qb, static_cast<const uint4*>(k));
+        } else {
+            const size_t smem = 2 * static_cast<size_t>(d.Hq) * kHeadDim * sizeof(float);
+            e0 = cudaFuncSetAttribute(k_dec_logits_any, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(smem));
+            if (e0 != cudaSuccess) return e0;
+            k_dec_logits_any<<<static_cast<unsigned>((n_cand + 127) / 128), 256, smem, st>>>(
+                a, qb, static_cast<const uint4*>(k));
+        }
+        k_dec_stats<<<d.Hq, 256, 0, st>>>(a, a.n_stat);
         k_dec_vote<<<static_cast<unsigned>((t + 1 + 255) / 256), 256, 0, st>>>(a);
         // top-k of the one-unit table [t, t + 1] kept in the cache, gated on the retrieval flag
         Derived du = d;

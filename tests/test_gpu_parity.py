@@ -676,6 +676,47 @@ def _decode_theta(qd, s_max):
     return best[0]
 
 
+@pytest.mark.parametrize("heads", [(6, 2), (8, 1), (4, 4), (16, 8)])
+def test_decode_group_sizes(heads):
+    """Retrieving decode steps for query-head groups of 3 (the kernel for any
+    group size), 8, 1 and 2 query heads per KV head: selection and output row
+    against the oracle."""
+    hq, hkv = heads
+    w, q, k, v, dev = inputs("gqa4-4k", n_tokens=2048, num_q_heads=hq, num_kv_heads=hkv, block_size=1,
+                             top_k=128, n_local=256, n_sink=32)
+    steps = np.arange(1900, 1906)
+    qd = _decode_queries(q, steps)
+    p = S.params_for(w, theta=2.0, max_cluster_subchunks=1)  # cos >= 2 never holds: every step retrieves
+    cache = torch.empty(S.scale_decode_cache_size(p), dtype=torch.uint8, device="cuda")
+    S.scale_decode_cache_init(cache)
+    ws = torch.empty(S.scale_decode_workspace_size(p), dtype=torch.uint8, device="cuda")
+    qd_dev = torch.from_numpy(qd).view(torch.bfloat16).cuda()
+    sel_full = np.full((w.n_tokens, w.top_k), -1, np.int32)
+    cnt_full = np.zeros(w.n_tokens, np.int32)
+    outs = []
+    for i, t in enumerate(steps):
+        out = torch.empty((hq, w.head_dim), dtype=torch.bfloat16, device="cuda")
+        S.scale_decode_step(p, int(t), qd_dev[i], dev[1], dev[2], cache, out, ws)
+        torch.cuda.synchronize()
+        assert S.decode_cache_state(cache)["retrieved"]
+        sel, cnt = S.decode_cache_selection(cache, p)
+        ref, gap = oracle.decode_select(qd[i], k, int(t), n_sink=w.n_sink, n_local=w.n_local, top_k=w.top_k)
+        assert cnt == len(ref)
+        if sel[:cnt].tolist() != ref.tolist():
+            assert gap < NEAR_TIE_GAP, f"step {t}: selection differs with gap {gap:.3e}"
+        sel_full[t, :cnt] = sel[:cnt]
+        cnt_full[t] = cnt
+        outs.append(to_f64_bf16(out))
+    q_rows = q.copy()
+    q_rows[steps] = qd
+    ref_attn = oracle.attention_rows(q=q_rows, k=k, v=v, sub_chunk=1, block_size=1, top_k=w.top_k,
+                                     n_sink=w.n_sink, n_local=w.n_local,
+                                     attn_scale=1.0 / np.sqrt(w.head_dim), per_subchunk=True,
+                                     unit_start=None, sel=sel_full, sel_count=cnt_full, rows=steps)
+    mx, mean = attn_errors(np.stack(outs), ref_attn)
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
 @pytest.mark.parametrize("theta", [-1.0, None])
 def test_decode_steps_with_selection_cache(theta):
     """scale_decode_step over 40 consecutive positions: reuse decisions, the
