@@ -702,6 +702,7 @@ def run_decode(args):
         p = S.params_for(w, theta=theta, max_cluster_subchunks=s_max)
         cache = torch.empty(S.scale_decode_cache_size(p), dtype=torch.uint8, device="cuda")
         ws = torch.empty(S.scale_decode_workspace_size(p), dtype=torch.uint8, device="cuda")
+        S.scale_workspace_init(ws)
         out = torch.empty((w.num_q_heads, w.head_dim), dtype=torch.bfloat16, device="cuda")
         for _ in range(max(1, args.warmup)):
             S.scale_decode_cache_init(cache)
@@ -716,6 +717,9 @@ def run_decode(args):
             ev[i + 1].record(stream)
         torch.cuda.synchronize()
         ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(n_steps)]
+        st = S.scale_get_device_status(ws)
+        if st != S.SCALE_OK:
+            raise RuntimeError(f"device status {st}: {S.status_string(st)}")
         res[label] = {"tpot_ms": statistics.mean(ms), "retrieving_step_ms": ms[0],
                       "reusing_step_ms": statistics.median(ms[1:]) if s_max > 1 else None,
                       "retrievals": -(-n_steps // s_max)}

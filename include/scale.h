@@ -292,7 +292,11 @@ int scale_sparse_prefill_paged(const scale_params_t *p, int32_t mode, int64_t to
  *   q_t, out_t  bf16 [H_q][128];  k, v  bf16 [n_tokens][H_kv][128]
  *   cache       scale_decode_cache_size() bytes, zeroed by
  *               scale_decode_cache_init() before the first step of a sequence
- *   ws          scale_decode_workspace_size() bytes (grows with n_tokens) */
+ *   ws          scale_decode_workspace_size() bytes (grows with n_tokens); its
+ *               first 256 bytes hold the device status word: zero them once
+ *               with scale_workspace_init(); a bounded wait of the step that
+ *               runs out records SCALE_ERR_TIMEOUT there, read with
+ *               scale_get_device_status(). */
 int scale_decode_cache_size(const scale_params_t *p, size_t *bytes);
 int scale_decode_cache_init(void *cache, size_t cache_bytes, scale_stream_t stream);
 int scale_decode_workspace_size(const scale_params_t *p, size_t *bytes);

@@ -610,7 +610,7 @@ int scale_decode_step(const scale_params_t* p, int64_t t, const void* q_t, const
     if (cache_bytes < decode_cache_bytes(d) || ws_bytes < decode_ws_bytes(d, decode_splits()))
         return SCALE_ERR_WORKSPACE;
     return cuda_status(launch_decode_step(d, t, q_t, k, v, static_cast<uint8_t*>(cache), out_t,
-                                          static_cast<uint8_t*>(ws), stream));
+                                          static_cast<uint8_t*>(ws), g_timeout_ns.load(), stream));
 }
 
 int scale_set_wait_timeout_ns(uint64_t ns)

@@ -23,10 +23,14 @@
 
 #include <cmath>
 
+#include "ptx_sm103.cuh"
 #include "scale_internal.h"
+#include "tma_host.h"
 
 namespace scale {
 namespace {
+
+using namespace scale_ptx;
 
 // Decode cache layout (bytes from its base).
 constexpr size_t kDecState = 0;     // int32[8]: valid, steps, retrieve, -, anchor position
@@ -65,8 +69,10 @@ struct DecArgs {
     float* scores;      // [cap]
     float* part;        // [H_q][splits][130]: max, sum, o[128]
     int splits;
-    float2* zpart;      // [H_q][n_stat] (max, sum) of each 64-candidate chunk
-    int n_stat;         // 64-candidate chunks of the candidates
+    float2* zpart;      // [H_q][n_stat] (max, sum) of each candidate chunk
+    int n_stat;         // candidate chunks (64 keys, or 128 for the tensor-core logits)
+    int32_t* status;    // device status word of the workspace
+    uint64_t timeout_ns;
 };
 
 __host__ __device__ __forceinline__ int64_t window_start(const DecArgs& a, int64_t t)
@@ -294,6 +300,203 @@ __global__ void __launch_bounds__(256) k_dec_logits_any(DecArgs a, const __nv_bf
     }
 }
 
+// Tensor-core form of the logits (g <= 16 query heads per KV head, H_kv <=
+// 16): a persistent CTA per SM walks its share of the items (128-key tile,
+// KV head j). Warp 0 lane 0 streams the tile's keys of head j by TMA (two
+// 64-dimension boxes of 128 rows, 32 KB, 128-byte swizzle) into a 4-stage
+// ring, so about 96 KB per SM are in flight without holding registers; warp 1
+// lane 0 issues D[key][row] = K_j . Q_j^T as eight tcgen05.mma (M = 128 keys,
+// N = 16: the g query rows of head j, then zero rows; K = 128) into one of two
+// 16-column TMEM accumulators; warps 2-5 read their 32 keys' columns, write
+// z = sigma * D for the live keys (W_t and beyond are dropped) and merge
+// each head's (max, sum of exp(z - max)) over the tile: a butterfly inside the
+// warp, then the four warps in TMEM-lane order. The query operand is written
+// to shared memory by the threads in the swizzled K-major layout the MMA
+// reads. Every wait is bounded; on expiry the kernel records
+// SCALE_ERR_TIMEOUT, drains what it issued and frees its TMEM.
+constexpr int kDtStages = 4;
+constexpr uint32_t kDtTile = 128 * 128 * 2;  // 128 keys x 128 dims (two 64-dim halves)
+constexpr uint32_t kDtHalf = kDtTile / 2;
+constexpr uint32_t kDtQ = 16 * 128 * 2;      // query rows of one KV head
+constexpr uint32_t kDtQHalf = kDtQ / 2;
+constexpr int kDtMaxHkv = 16;
+constexpr uint32_t kDtSmem = kDtStages * kDtTile + kDtMaxHkv * kDtQ + 1024;
+constexpr int kDtThreads = 192;
+static_assert(kDtSmem <= 227 * 1024 - 1024, "tensor-core decode logits shared memory");
+
+struct DtBars {
+    uint64_t k_full[kDtStages], k_empty[kDtStages];
+    uint64_t d_full[2], d_empty[2];
+    uint64_t drain;
+};
+
+__device__ __forceinline__ void dt_fail(volatile int* abort_flag, int32_t* status)
+{
+    *abort_flag = 1;
+    record_status(status, SCALE_ERR_TIMEOUT);
+}
+
+template <int G>
+__global__ void __launch_bounds__(kDtThreads, 1)
+k_dec_logits_tc(const __grid_constant__ CUtensorMap tk, const DecArgs a, const __nv_bfloat16* __restrict__ q)
+{
+    if (!a.state[2]) return;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ DtBars bars;
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+    __shared__ float2 s_stat[2][4][G];
+    const int64_t lo = a.n_sink, hi = window_start(a, a.t);
+    const int64_t items = (hi - lo + 127) / 128 * a.Hkv;
+    const int64_t i0 = items * blockIdx.x / gridDim.x, i1 = items * (blockIdx.x + 1) / gridDim.x;
+    if (i1 <= i0) return;
+    const int n_it = static_cast<int>(i1 - i0);
+    uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+    uint8_t* kbuf = smem;
+    uint8_t* qbuf = smem + kDtStages * kDtTile;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    // query operand: row r of head j is query head j G + r (zero for r >= G);
+    // 16-byte chunk c of a 128-byte row goes to chunk c ^ (row % 8)
+    for (int x = tid; x < a.Hkv * 16 * 16; x += blockDim.x) {
+        const int c = x & 15, r = (x >> 4) & 15, j = x >> 8;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (r < G) val = *reinterpret_cast<const uint4*>(q + (static_cast<int64_t>(j) * G + r) * kHeadDim + 8 * c);
+        const int hf = c >> 3, cc = c & 7;
+        *reinterpret_cast<uint4*>(qbuf + j * kDtQ + hf * kDtQHalf + (r >> 3) * 1024 + (r & 7) * 128 +
+                                  ((cc ^ (r & 7)) << 4)) = val;
+    }
+    fence_proxy_async_smem();
+    if (tid == 0) {
+        abort_flag = 0;
+        for (int i = 0; i < kDtStages; ++i) {
+            mbar_init(&bars.k_full[i], 1);
+            mbar_init(&bars.k_empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&bars.d_full[i], 1);
+            mbar_init(&bars.d_empty[i], 128);
+        }
+        mbar_init(&bars.drain, 1);
+        fence_barrier_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_slot, 32);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tk);
+            int issued[kDtStages] = {};
+            for (int it = 0; it < n_it && !abort_flag; ++it) {
+                const int st = it % kDtStages;
+                if (it >= kDtStages &&
+                    !mbar_wait_bounded(&bars.k_empty[st], ((it / kDtStages) - 1) & 1, a.timeout_ns, &abort_flag)) {
+                    dt_fail(&abort_flag, a.status);
+                    break;
+                }
+                const int64_t item = i0 + it;
+                const int64_t tile = item / a.Hkv;
+                const int j = static_cast<int>(item - tile * a.Hkv);
+                const int32_t key0 = static_cast<int32_t>(lo + 128 * tile);
+                mbar_arrive_expect_tx(&bars.k_full[st], kDtTile);
+                ++issued[st];
+                for (int hf = 0; hf < 2; ++hf)
+                    tma_load_3d(kbuf + st * kDtTile + hf * kDtHalf, &tk, &bars.k_full[st], hf * 64, j, key0);
+            }
+            if (abort_flag)
+                for (int st = 0; st < kDtStages; ++st)
+                    if (issued[st]) mbar_wait_bounded(&bars.k_full[st], (issued[st] - 1) & 1, a.timeout_ns, nullptr);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, 16, 0);
+            const uint64_t kdesc0 = sdesc_sw128(smem_addr(kbuf), 16, 1024);
+            const uint64_t qdesc0 = sdesc_sw128(smem_addr(qbuf), 16, 1024);
+            bool ok = true;
+            for (int it = 0; it < n_it; ++it) {
+                const int st = it % kDtStages, b = it & 1;
+                if (!mbar_wait_bounded(&bars.k_full[st], (it / kDtStages) & 1, a.timeout_ns, &abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                if (it >= 2 && !mbar_wait_bounded(&bars.d_empty[b], ((it >> 1) - 1) & 1, a.timeout_ns, &abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int64_t item = i0 + it;
+                const int j = static_cast<int>(item - item / a.Hkv * a.Hkv);
+                mma_ss_k128_ab<kDtHalf, kDtQHalf>(tmem + b * 16, kdesc0 + st * (kDtTile >> 4),
+                                                  qdesc0 + j * (kDtQ >> 4), idesc, 0u);
+                mma_commit(&bars.d_full[b]);
+                mma_commit(&bars.k_empty[st]);
+            }
+            if (!ok) {
+                dt_fail(&abort_flag, a.status);
+                mma_commit(&bars.drain);
+                mbar_wait_bounded(&bars.drain, 0, a.timeout_ns, nullptr);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        // Every epilogue warp runs one named barrier per item, also after a
+        // failed wait (it then skips the work).
+        const int qq = warp & 3;  // TMEM lane quarter this warp may access
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(qq * 32) << 16);
+        bool ok = true;
+        for (int it = 0; it < n_it; ++it) {
+            const int b = it & 1;
+            const int64_t item = i0 + it;
+            const int64_t tile = item / a.Hkv;
+            const int j = static_cast<int>(item - tile * a.Hkv);
+            if (ok) {
+                ok = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.d_full[b], (it >> 1) & 1, a.timeout_ns, &abort_flag));
+                if (ok) {
+                    tc_fence_after();
+                    uint32_t r[16];
+                    tmem_ld16(lane_base + b * 16, r);
+                    tmem_ld_wait();
+                    tc_fence_before();
+                    mbar_arrive(&bars.d_empty[b]);
+                    const int64_t key = lo + 128 * tile + qq * 32 + lane;
+                    const bool live = key < hi;
+#pragma unroll
+                    for (int hl = 0; hl < G; ++hl) {
+                        const float zv = a.sigma * __uint_as_float(r[hl]);
+                        if (live) a.z[static_cast<int64_t>(j * G + hl) * a.cap + key] = zv;
+                        float m = live ? zv : -INFINITY, sum = live ? 1.f : 0.f;
+                        for (int o = 1; o < 32; o <<= 1)
+                            merge_ms(m, sum, __shfl_xor_sync(0xFFFFFFFFu, m, o), __shfl_xor_sync(0xFFFFFFFFu, sum, o));
+                        if (lane == 0) s_stat[b][qq][hl] = make_float2(m, sum);
+                    }
+                }
+            }
+            named_barrier(1, 128);
+            if (ok && qq == 0 && lane < G) {
+                float2 t = s_stat[b][0][lane];
+                for (int w = 1; w < 4; ++w) merge_ms(t.x, t.y, s_stat[b][w][lane].x, s_stat[b][w][lane].y);
+                a.zpart[static_cast<int64_t>(j * G + lane) * a.n_stat + tile] = t;
+            }
+        }
+        if (!ok) dt_fail(&abort_flag, a.status);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 32);
+    }
+}
+
 // Fixed-order block reductions (warp butterflies, then the warps in order).
 __device__ __forceinline__ float block_max256(float v, float* red)
 {
@@ -501,7 +704,7 @@ size_t decode_ws_bytes(const Derived& d, int splits)
 int decode_splits() { return kDecSplits; }
 
 cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const void* k, const void* v,
-                               uint8_t* cache, void* out, uint8_t* ws, cudaStream_t st)
+                               uint8_t* cache, void* out, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st)
 {
     DecArgs a;
     a.Hq = d.Hq;
@@ -522,6 +725,8 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
     a.sel = reinterpret_cast<int32_t*>(cache + kDecAnchor + static_cast<size_t>(d.Hq) * kHeadDim * sizeof(float));
     a.sel_count = a.sel + (d.k > 0 ? d.k : 1);
     a.splits = kDecSplits;
+    a.status = reinterpret_cast<int32_t*>(ws + kStatusOffset);
+    a.timeout_ns = timeout_ns;
     size_t off = 256;
     auto take = [&](size_t bytes) {
         const size_t at = off;
@@ -542,9 +747,26 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
     k_dec_gate<<<1, 256, 0, st>>>(a, qb);
     const int64_t n_cand = window_start(a, t) - d.n_sink;
     if (n_cand > 0) {
-        a.n_stat = static_cast<int>((n_cand + kDecStat - 1) / kDecStat);
         cudaError_t e0;
-        if (d.g == 1 || d.g == 2 || d.g == 4 || d.g == 8) {
+        if ((d.g == 1 || d.g == 2 || d.g == 4 || d.g == 8) && d.Hkv <= kDtMaxHkv) {
+            // tensor cores, keys streamed by TMA
+            const int64_t tiles = (n_cand + 127) / 128;
+            a.n_stat = static_cast<int>(tiles);
+            CUtensorMap tk;
+            if (!scale_host::make_token_major_map(&tk, k, kHeadDim, d.Hkv, d.N, 64, 128)) return cudaErrorInvalidValue;
+            int dev = 0, sms = 0;
+            e0 = cudaGetDevice(&dev);
+            if (e0 == cudaSuccess) e0 = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            if (e0 != cudaSuccess) return e0;
+            const int64_t items = tiles * d.Hkv;
+            const unsigned grid = static_cast<unsigned>(items < sms ? items : sms);
+            auto kern = d.g == 1 ? k_dec_logits_tc<1> : d.g == 2 ? k_dec_logits_tc<2>
+                      : d.g == 4 ? k_dec_logits_tc<4> : k_dec_logits_tc<8>;
+            e0 = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kDtSmem));
+            if (e0 != cudaSuccess) return e0;
+            kern<<<grid, kDtThreads, kDtSmem, st>>>(tk, a, qb);
+        } else if (d.g == 1 || d.g == 2 || d.g == 4 || d.g == 8) {
+            a.n_stat = static_cast<int>((n_cand + kDecStat - 1) / kDecStat);
             auto kern = d.g == 1 ? k_dec_logits<1> : d.g == 2 ? k_dec_logits<2> : d.g == 4 ? k_dec_logits<4>
                                                                                          : k_dec_logits<8>;
             const size_t smem = static_cast<size_t>(d.Hq) * kHeadDim * sizeof(float);
@@ -553,6 +775,7 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
             kern<<<static_cast<unsigned>((n_cand + kDecBlockKeys - 1) / kDecBlockKeys), 256, smem, st>>>(
                 a, qb, static_cast<const uint4*>(k));
         } else {
+            a.n_stat = static_cast<int>((n_cand + kDecStat - 1) / kDecStat);
             const size_t smem = 2 * static_cast<size_t>(d.Hq) * kHeadDim * sizeof(float);
             e0 = cudaFuncSetAttribute(k_dec_logits_any, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       static_cast<int>(smem));

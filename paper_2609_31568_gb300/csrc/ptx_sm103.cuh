@@ -205,6 +205,44 @@ __device__ __forceinline__ void mma_ss_k128(uint32_t d_tmem, uint64_t a_desc, ui
         : "memory");
 }
 
+// mma_ss_k128 for operands whose second 64-column half lies at different
+// offsets: `a_half` bytes after the first for A, `b_half` for B.
+template <uint32_t a_half, uint32_t b_half>
+__device__ __forceinline__ void mma_ss_k128_ab(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                               uint32_t idesc, uint32_t accumulate)
+{
+    constexpr uint64_t ha = a_half >> 4, hb = b_half >> 4;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t.reg .b64 a, b;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "setp.ne.b32 q, %5, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t"
+        "add.s64 a, %1, 2;\n\tadd.s64 b, %2, 2;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, 4;\n\tadd.s64 b, %2, 4;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, 6;\n\tadd.s64 b, %2, 6;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %6;\n\tadd.s64 b, %2, %10;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %7;\n\tadd.s64 b, %2, %11;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %8;\n\tadd.s64 b, %2, %12;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t"
+        "add.s64 a, %1, %9;\n\tadd.s64 b, %2, %13;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %3, q;\n\t}" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate), "r"(1u), "n"(ha), "n"(ha + 2),
+        "n"(ha + 4), "n"(ha + 6), "n"(hb), "n"(hb + 2), "n"(hb + 4), "n"(hb + 6)
+        : "memory");
+}
+
+// Order this thread's generic-proxy shared-memory writes before later
+// async-proxy reads of them (a tcgen05.mma operand written with st.shared).
+__device__ __forceinline__ void fence_proxy_async_smem()
+{
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Eight MMAs D (+)= A_j * B_j, j = 0..7, with A in TMEM (8 columns of packed
 // bf16 pairs = 16 K elements per step) and B an MN-major smem operand whose
 // descriptor advances by `step_bytes` per 16-element K step.

@@ -194,7 +194,7 @@ size_t decode_cache_bytes(const Derived& d);
 size_t decode_ws_bytes(const Derived& d, int splits);
 int decode_splits();
 cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const void* k, const void* v,
-                               uint8_t* cache, void* out, uint8_t* ws, cudaStream_t st);
+                               uint8_t* cache, void* out, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 
 // Packed distant rows per (unit, KV head) at block size 1: n_sink + k rounded
 // up to a multiple of 128.

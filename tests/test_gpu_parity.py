@@ -676,11 +676,12 @@ def _decode_theta(qd, s_max):
     return best[0]
 
 
-@pytest.mark.parametrize("heads", [(6, 2), (8, 1), (4, 4), (16, 8)])
+@pytest.mark.parametrize("heads", [(6, 2), (8, 1), (4, 4), (16, 8), (34, 17)])
 def test_decode_group_sizes(heads):
-    """Retrieving decode steps for query-head groups of 3 (the kernel for any
-    group size), 8, 1 and 2 query heads per KV head: selection and output row
-    against the oracle."""
+    """Retrieving decode steps for query-head groups of 3 (the CUDA-core kernel
+    for any group size), 8, 1 and 2 query heads per KV head (tensor cores), and
+    2 with 17 KV heads (the register-blocked CUDA-core kernel): selection and
+    output row against the oracle."""
     hq, hkv = heads
     w, q, k, v, dev = inputs("gqa4-4k", n_tokens=2048, num_q_heads=hq, num_kv_heads=hkv, block_size=1,
                              top_k=128, n_local=256, n_sink=32)
@@ -690,6 +691,7 @@ def test_decode_group_sizes(heads):
     cache = torch.empty(S.scale_decode_cache_size(p), dtype=torch.uint8, device="cuda")
     S.scale_decode_cache_init(cache)
     ws = torch.empty(S.scale_decode_workspace_size(p), dtype=torch.uint8, device="cuda")
+    S.scale_workspace_init(ws)
     qd_dev = torch.from_numpy(qd).view(torch.bfloat16).cuda()
     sel_full = np.full((w.n_tokens, w.top_k), -1, np.int32)
     cnt_full = np.zeros(w.n_tokens, np.int32)
@@ -707,6 +709,7 @@ def test_decode_group_sizes(heads):
         sel_full[t, :cnt] = sel[:cnt]
         cnt_full[t] = cnt
         outs.append(to_f64_bf16(out))
+    assert S.scale_get_device_status(ws) == S.SCALE_OK
     q_rows = q.copy()
     q_rows[steps] = qd
     ref_attn = oracle.attention_rows(q=q_rows, k=k, v=v, sub_chunk=1, block_size=1, top_k=w.top_k,
@@ -731,6 +734,7 @@ def test_decode_steps_with_selection_cache(theta):
     cache = torch.empty(S.scale_decode_cache_size(p), dtype=torch.uint8, device="cuda")
     S.scale_decode_cache_init(cache)
     ws = torch.empty(S.scale_decode_workspace_size(p), dtype=torch.uint8, device="cuda")
+    S.scale_workspace_init(ws)
     qd_dev = torch.from_numpy(qd).view(torch.bfloat16).cuda()
     want_r, anchor_of, margin = oracle.decode_reuse(qd, theta, s_max)
     assert margin > 1e-5
@@ -761,6 +765,7 @@ def test_decode_steps_with_selection_cache(theta):
                                      n_sink=w.n_sink, n_local=w.n_local,
                                      attn_scale=1.0 / np.sqrt(w.head_dim), per_subchunk=True,
                                      unit_start=None, sel=sel_full, sel_count=cnt_full, rows=steps)
+    assert S.scale_get_device_status(ws) == S.SCALE_OK
     mx, mean = attn_errors(np.stack(outs), ref_attn)
     print(f"theta={theta:.4f}: {int(want_r.sum())} retrievals in {len(steps)} steps, {near} near-ties, "
           f"attention max {mx:.3e} mean {mean:.3e}")
