@@ -177,18 +177,25 @@ __device__ __forceinline__ uint32_t float_key(float f)
 constexpr int kTopkThreads = 1024;
 constexpr int kTopkUnroll = 16;  // independent loads in flight per thread
 
-// One CTA per unit. The k-th largest key T is found with four 8-bit radix
-// passes (16 coalesced loads in flight per thread); the selected blocks are
-// those with key > T plus the lowest-indexed ones with key == T, emitted in
-// ascending block order: every warp owns a contiguous segment, counts its
-// picks, and after one scan over the warps writes them in order with
-// warp-level prefix sums.
+constexpr int kSortMax = 4096;     // candidates up to which k_topk sorts instead
+
+// One CTA per unit. Up to kSortMax candidates, a bitonic sort in shared
+// memory of the 64-bit keys (~float_key(score), index) puts the picks first
+// (higher score first, equal scores by lower index); their indices are marked
+// in a bitmap and written in ascending order after one scan. Beyond that, the
+// k-th largest key T is found with four 8-bit radix passes (16 coalesced
+// loads in flight per thread); the selected blocks are those with key > T
+// plus the lowest-indexed ones with key == T, emitted in ascending block
+// order: every warp owns a contiguous segment, counts its picks, and after
+// one scan over the warps writes them in order with warp-level prefix sums.
+// Both give the same selection.
 __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* __restrict__ scores,
                                                        int32_t* __restrict__ sel,
                                                        int32_t* __restrict__ sel_count)
 {
     __shared__ int hist[256];
-    __shared__ int whist[kTopkThreads / 32][256];  // per-warp histograms
+    __shared__ __align__(16) int whist[kTopkThreads / 32][256];  // per-warp histograms, or the sort keys
+    static_assert(sizeof(whist) >= kSortMax * sizeof(uint64_t), "sort buffer");
     __shared__ uint32_t s_prefix;
     __shared__ int s_need;
     if (a.gate && !*a.gate) return;
@@ -209,12 +216,66 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
         if (threadIdx.x == 0) sel_count[u] = static_cast<int32_t>(n);
         return;
     }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (n <= kSortMax) {
+        uint64_t* sk = reinterpret_cast<uint64_t*>(&whist[0][0]);
+        int np = 1;
+        while (np < n) np <<= 1;
+        for (int i = threadIdx.x; i < np; i += blockDim.x)
+            sk[i] = i < n ? (static_cast<uint64_t>(~float_key(sc[lo + i])) << 32) | static_cast<uint32_t>(i)
+                          : ~0ull;  // padding sorts last
+        __syncthreads();
+        for (int size = 2; size <= np; size <<= 1)
+            for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                for (int i = threadIdx.x; i < np; i += blockDim.x) {
+                    const int l = i ^ stride;
+                    if (l > i) {
+                        const uint64_t x = sk[i], y = sk[l];
+                        if ((x > y) == ((i & size) == 0)) {
+                            sk[i] = y;
+                            sk[l] = x;
+                        }
+                    }
+                }
+                __syncthreads();
+            }
+        uint32_t* bm = reinterpret_cast<uint32_t*>(hist);  // np / 32 <= 128 words
+        for (int w = threadIdx.x; w < np / 32 + 1; w += blockDim.x) bm[w] = 0u;
+        __syncthreads();
+        for (int r = threadIdx.x; r < a.k; r += blockDim.x) {
+            const uint32_t i = static_cast<uint32_t>(sk[r]);
+            atomicOr(&bm[i >> 5], 1u << (i & 31));
+        }
+        __syncthreads();
+        // ascending output: word t of the bitmap to thread t, exclusive scan of the counts
+        __shared__ int s_wsum[4];
+        const int nwords = (np + 31) / 32;
+        uint32_t word = threadIdx.x < nwords ? bm[threadIdx.x] : 0u;
+        const int c = __popc(word);
+        int inc = c;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+            if (lane >= o) inc += y;
+        }
+        if (lane == 31 && warp < 4) s_wsum[warp] = inc;
+        __syncthreads();
+        if (threadIdx.x < nwords) {
+            int p = inc - c;
+            for (int w = 0; w < warp; ++w) p += s_wsum[w];
+            while (word) {
+                const int bit = __ffs(word) - 1;
+                word &= word - 1;
+                out[p++] = static_cast<int32_t>(lo + 32 * threadIdx.x + bit);
+            }
+        }
+        if (threadIdx.x == 0) sel_count[u] = a.k;  // n > k: exactly k picks
+        return;
+    }
     if (threadIdx.x == 0) {
         s_prefix = 0;
         s_need = a.k;
     }
     uint32_t mask = 0;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int shift = 24; shift >= 0; shift -= 8) {
         for (int i = threadIdx.x; i < (kTopkThreads / 32) * 256; i += blockDim.x) (&whist[0][0])[i] = 0;
         __syncthreads();
