@@ -563,7 +563,7 @@ __global__ void __launch_bounds__(256) k_dec_vote(DecArgs a)
 // cached selection (produced by the top-k: ascending, inside [n_sink, W_a)
 // with W_a <= W_t), then the window [W_t, t]. One warp per query head of KV
 // head blockIdx.x, lane l holding dimensions [4 l, 4 l + 4); online softmax in
-// log2 units, four keys per update (their loads and dot products are
+// log2 units, eight keys per update (their loads and dot products are
 // independent, so they overlap). Writes (max, sum, unnormalised o) per
 // (head, split).
 __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16* __restrict__ q,
@@ -587,42 +587,50 @@ __global__ void __launch_bounds__(256) k_dec_attn(DecArgs a, const __nv_bfloat16
     auto key = [&](int i) -> int64_t {
         return i < n_s ? i : (i < n_s + n_sel ? a.sel[i - n_s] : W + (i - n_s - n_sel));
     };
+    constexpr int KB = 8;  // keys per update
     int i = i0;
-    for (; i + 4 <= i1; i += 4) {
-        uint2 kw[4], vw[4];
+    for (; i + KB <= i1; i += KB) {
+        uint2 kw[KB], vw[KB];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < KB; ++u) {
             const int64_t row = (key(i + u) * a.Hkv + j) * 32 + lane;
             kw[u] = k[row];
             vw[u] = v[row];
         }
-        float s[4];
+        float s[KB];
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
+        for (int u = 0; u < KB; ++u)
             s[u] = q0 * bf16_lo(kw[u].x) + q1 * bf16_hi(kw[u].x) + q2 * bf16_lo(kw[u].y) + q3 * bf16_hi(kw[u].y);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-            for (int u = 0; u < 4; ++u) s[u] += __shfl_xor_sync(0xFFFFFFFFu, s[u], o);
+            for (int u = 0; u < KB; ++u) s[u] += __shfl_xor_sync(0xFFFFFFFFu, s[u], o);
         float m_new = m;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < KB; ++u) {
             s[u] *= a.attn_scale_log2;
             m_new = fmaxf(m_new, s[u]);
         }
         const float alpha = exp2f(m - m_new);
-        float p[4];
+        float p[KB], psum = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) p[u] = exp2f(s[u] - m_new);
-        l = l * alpha + (((p[0] + p[1]) + p[2]) + p[3]);
-        o0 = o0 * alpha + p[0] * bf16_lo(vw[0].x) + p[1] * bf16_lo(vw[1].x) + p[2] * bf16_lo(vw[2].x) +
-             p[3] * bf16_lo(vw[3].x);
-        o1 = o1 * alpha + p[0] * bf16_hi(vw[0].x) + p[1] * bf16_hi(vw[1].x) + p[2] * bf16_hi(vw[2].x) +
-             p[3] * bf16_hi(vw[3].x);
-        o2 = o2 * alpha + p[0] * bf16_lo(vw[0].y) + p[1] * bf16_lo(vw[1].y) + p[2] * bf16_lo(vw[2].y) +
-             p[3] * bf16_lo(vw[3].y);
-        o3 = o3 * alpha + p[0] * bf16_hi(vw[0].y) + p[1] * bf16_hi(vw[1].y) + p[2] * bf16_hi(vw[2].y) +
-             p[3] * bf16_hi(vw[3].y);
+        for (int u = 0; u < KB; ++u) {
+            p[u] = exp2f(s[u] - m_new);
+            psum += p[u];
+        }
+        l = l * alpha + psum;
+        float d0 = 0.f, d1 = 0.f, d2 = 0.f, d3 = 0.f;
+#pragma unroll
+        for (int u = 0; u < KB; ++u) {
+            d0 += p[u] * bf16_lo(vw[u].x);
+            d1 += p[u] * bf16_hi(vw[u].x);
+            d2 += p[u] * bf16_lo(vw[u].y);
+            d3 += p[u] * bf16_hi(vw[u].y);
+        }
+        o0 = o0 * alpha + d0;
+        o1 = o1 * alpha + d1;
+        o2 = o2 * alpha + d2;
+        o3 = o3 * alpha + d3;
         m = m_new;
     }
     for (; i < i1; ++i) {
