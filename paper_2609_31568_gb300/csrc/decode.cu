@@ -15,10 +15,11 @@
 //    have shared it, and retrieves (and becomes the anchor) otherwise;
 //  - attention (Eq. 10 for one row): keys = sinks U selection U [W_t, t].
 //
-// Scoring one query against every key is a matrix-vector product: it runs on
-// the CUDA cores, one thread per key, reading K once in 16-byte pieces (the
-// step is bound by HBM, not by arithmetic). Whether the step retrieves is
-// decided on the device, so a step never synchronises with the host.
+// Scoring one query against every key is a matrix-vector product per KV head,
+// bound by reading K once: k_dec_logits_tc streams the keys by TMA and runs
+// the products on the tensor cores; shapes it does not cover use CUDA-core
+// kernels. Whether the step retrieves is decided on the device, so a step
+// never synchronises with the host.
 #include <cuda_bf16.h>
 
 #include <cmath>
