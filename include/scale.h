@@ -10,7 +10,8 @@
  *
  *   scale_build_reps      (a) block representative keys, sub-chunk
  *                             fingerprints (Eq. 6) and anchor-based clusters
- *                             (Eq. 8, Algorithm 1);
+ *                             (Eq. 8, Algorithm 1); scale_build_reps_range
+ *                             does the same chunk by chunk;
  *   scale_select          (b) GQA-aware scoring of the representatives against
  *                             each cluster's anchor fingerprint with head
  *                             soft-voting, and (c) a deterministic top-k

@@ -5,8 +5,11 @@
 //   k_logits  z[u][h][b] = sigma * v_a(u)^(h) . r_b^(h/g)   (fp32 GEMM tile per KV head)
 //   k_stats   per (u, h): max_b z and 1 / sum_b exp(z - max) over the candidates
 //   k_vote    score[u][b] = sum_h exp(z[u][h][b] - max) / sum   (heads in order)
-//   k_topk    radix select of the k-th largest (score, -b) key, then an
-//             index-ordered compaction: output ascending, ties to the lower b.
+//   k_topk    up to 4096 candidates a bitonic sort of (score, -b) keys in
+//             shared memory, beyond that a radix select of the k-th largest
+//             key and an index-ordered compaction (and, with a scratch area
+//             and more than 64K candidates, the multi-CTA form below): output
+//             ascending, ties to the lower b.
 //
 // Candidates of unit u are the blocks with a token in [n_sink, W_u),
 // W_u = max(0, s_u - n_local): the contiguous range [b_lo, b_hi(u)).
