@@ -38,6 +38,8 @@
  *    _host), 16-byte aligned, owned by the caller. The library allocates no
  *    memory on any path; scratch lives in a caller-provided workspace of
  *    scale_workspace_size() bytes, initialised once with scale_workspace_init().
+ *    (scale_prefill_host creates, for the duration of the call, two streams
+ *    and their events to overlap its copies with the compute.)
  *  - Streams. `stream` is a cudaStream_t (NULL = legacy default stream). Calls
  *    only enqueue work on it and never synchronise, except the functions
  *    documented as synchronous (scale_get_device_status, scale_prefill_host).
