@@ -203,4 +203,18 @@ def test_paged_entry_points_validate_before_launch(lib, page_size, over, rc):
                                           None, None, None, None, None, 0, None) == rc
     assert lib.scale_build_reps_paged(ctypes.byref(p), None, ctypes.byref(kv), None, None, None, None,
                                       None, 0, None) == rc
+    assert lib.scale_build_reps_range_paged(ctypes.byref(p), 0, p.outer_chunk, None, ctypes.byref(kv), None,
+                                            None, None, None, None, 0, None) == rc
+
+
+@pytest.mark.parametrize("over,tb,te,rc", [
+    (dict(head_dim=64), 0, 8192, S.SCALE_ERR_UNSUPPORTED),   # parameters are checked first
+    ({}, 0, 8192, S.SCALE_ERR_INVALID_ARG),                  # valid range, null pointers
+    ({}, 4096, 8192, S.SCALE_ERR_INVALID_ARG),               # not on an outer-chunk boundary
+    ({}, 8192, 4096, S.SCALE_ERR_INVALID_ARG),
+])
+def test_range_build_validates_before_launch(lib, over, tb, te, rc):
+    p = _p(**over)
+    assert lib.scale_build_reps_range(ctypes.byref(p), tb, te, None, None, None, None, None, None, None, 0,
+                                      None) == rc
 
