@@ -623,6 +623,30 @@ def test_paged_kv_equals_contiguous(name, over, page, mode):
     assert torch.equal(buf.out, ref.out)
 
 
+@pytest.mark.parametrize("name,over,page", [("gqa4-4k", dict(n_tokens=3000), 128),
+                                            ("llama8b-32k", dict(n_tokens=20000), 256)])
+def test_paged_range_build_equals_contiguous(name, over, page):
+    """scale_build_reps_range_paged over the outer chunks in order, on a
+    shuffled page pool, gives the contiguous whole-sequence step (a) bit for
+    bit: representatives, fingerprints and the appended unit table."""
+    w, q, k, v, dev = inputs(name, **over)
+    p, ref = gpu_path(w, PER_CLUSTER, dev, want_scores=False)
+    kp, table = _paged(dev[1], page, np.random.default_rng(5))
+    vp, _ = _paged(dev[2], page, np.random.default_rng(5))
+    kv = S.kv_pages(kp, vp, table, page)
+    buf = S.allocate(p, PER_CLUSTER)
+    for t0 in range(0, w.n_tokens, w.outer_chunk):
+        t1 = min(w.n_tokens, t0 + w.outer_chunk)
+        S.scale_build_reps_range_paged(p, t0, t1, dev[0], kv, buf.reps, buf.fingerprints, buf.unit_start,
+                                       buf.n_units, buf.ws)
+    torch.cuda.synchronize()
+    assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
+    assert torch.equal(buf.reps.view(torch.int32), ref.reps.view(torch.int32))
+    assert torch.equal(buf.fingerprints.view(torch.int32), ref.fingerprints.view(torch.int32))
+    assert torch.equal(buf.unit_start, ref.unit_start)
+    assert int(buf.n_units.item()) == int(ref.n_units.item())
+
+
 def test_paged_kv_entry_outside_pool_reads_zeros():
     """A page-table entry outside the pool is not dereferenced; its tokens act
     as zero keys and values (checked against the contiguous path with those
