@@ -379,3 +379,40 @@ def test_key_set_revealed_by_uniform_attention():
         want = np.zeros(N)
         want[ks] = 1.0 / len(ks)
         np.testing.assert_allclose(out[i, 0], want, rtol=0, atol=1e-15, err_msg=f"row {p}")
+
+
+def test_member_selection_uses_member_j_against_the_cluster_candidates():
+    """Sec. IV-C's per-member retrieval by construction: block b's
+    representative is the unit vector e_b, and a sub-chunk's fingerprint
+    points at one block with a large weight in every head, so with top_k = 1
+    the selection is that block. Member j of the cluster [8, 12) must pick the
+    block its own fingerprint names (not the anchor's, nor a neighbour's), from
+    the cluster's candidates (blocks before W_u = 8 * 64 - 64 = 448, i.e. 0..27,
+    not the member's own later range); clusters of one sub-chunk keep their
+    anchor."""
+    from types import SimpleNamespace
+
+    L, B, nb, Hq = 64, 16, 64, 2
+    w = SimpleNamespace(num_q_heads=Hq, n_tokens=16 * L, sub_chunk=L, block_size=B, top_k=1, n_sink=0,
+                        n_local=L)
+    reps = np.zeros((1, nb, 128))
+    for b in range(nb):
+        reps[0, b, b] = 1.0
+    v = np.zeros((16, Hq * 128))
+    target = {8: 5, 9: 20, 10: 17, 11: 30, 3: 2}  # sub-chunk -> block its fingerprint names
+    for i, b in target.items():
+        for h in range(Hq):
+            v[i, h * 128 + b] = 50.0
+    unit_start = np.array(list(range(9)) + [12, 13, 14, 15, 16], np.int32)  # cluster [8, 12) is unit 8
+    anchor = oracle.member_selection(w, reps, v, unit_start, 0)
+    assert anchor["sel"][8].tolist() == [5]
+    assert oracle.member_selection(w, reps, v, unit_start, 1)["sel"][8].tolist() == [20]
+    assert oracle.member_selection(w, reps, v, unit_start, 2)["sel"][8].tolist() == [17]
+    # member 3 names block 30: inside its own per-sub-chunk range (blocks < 40) but
+    # not the cluster's (blocks < 28), so it must not be selected
+    m3 = oracle.member_selection(w, reps, v, unit_start, 3)
+    assert m3["cand_count"][8] == 28 and 0 <= m3["sel"][8][0] < 28
+    for j in (1, 2, 3):  # singleton units keep their anchor's selection
+        r = oracle.member_selection(w, reps, v, unit_start, j)
+        assert r["sel"][3].tolist() == anchor["sel"][3].tolist() == [2]
+        assert r["sel"][0].tolist() == anchor["sel"][0].tolist()
