@@ -159,8 +159,13 @@ int scale_build_reps_range(const scale_params_t *p, int64_t tok_begin, int64_t t
  *  - Set-up: the first call on each device looks up the array's device address
  *    with that device current; make that first call before any stream capture.
  *  - Sharing: every call on a device uses the same array, which keeps the last
- *    call's contents; calls whose work overlaps on the GPU (other streams, or
- *    other host threads) race on it and must be serialised by the caller. */
+ *    call's contents (step (a) writes each scratch element before reading it,
+ *    so nothing is cleared between calls); calls whose work overlaps on the
+ *    GPU (other streams, or other host threads) race on it and must be
+ *    serialised by the caller.
+ *  - Errors: argument checks as for scale_build_reps, returned synchronously.
+ *    There is no device status to read: step (a)'s kernels have no bounded
+ *    waits or device-side checks and record none. */
 int scale_build_reps_noalloc(const scale_params_t *p, const void *q, const void *k, float *reps,
                              float *fingerprints, int32_t *unit_start, int32_t *n_units,
                              scale_stream_t stream);

@@ -77,10 +77,10 @@ extern "C" int scale_build_reps_noalloc(const scale_params_t* p, const void* q, 
     void* scratch = nullptr;
     if ((rc = scratch_address(&scratch))) return rc;
     // The array keeps the previous call's contents. Step (a) writes every
-    // scratch element before reading it; the status word at its start is
-    // cleared so that it never reports an earlier call's state.
-    if (cudaMemsetAsync(static_cast<uint8_t*>(scratch) + kStatusOffset, 0, 256, stream) != cudaSuccess)
-        return SCALE_ERR_CUDA;
+    // scratch element before reading it, so nothing needs clearing; its
+    // kernels record no device status (they have no bounded waits and no
+    // device-side checks), so the status word at the array's start is never
+    // written or read.
     const KvPaging pg{nullptr, 0, 0, d.N, d.N};
     return launch_build_reps(d, q, k, pg, reps, fingerprints, unit_start, n_units,
                              static_cast<uint8_t*>(scratch), stream) == cudaSuccess

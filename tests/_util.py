@@ -61,6 +61,17 @@ def compare_selection(gpu_sel: np.ndarray, gpu_cnt: np.ndarray, ref: dict):
     return same, differ_near
 
 
+def selection_for_reference(gpu_sel: np.ndarray, ref: dict, same: np.ndarray) -> np.ndarray:
+    """The selection the attention reference runs on: the oracle's for every
+    unit whose GPU selection matches it, the GPU's own for the units that
+    differ at a near-tie (both are correct selections there, and the
+    attention must be right for the one the path actually used)."""
+    k = ref["sel"].shape[1]
+    merged = np.array(ref["sel"], np.int32, copy=True)
+    merged[~same] = gpu_sel[~same, :k]
+    return merged
+
+
 def attn_errors(gpu: np.ndarray, ref: np.ndarray):
     d = np.abs(gpu - ref)
     return float(d.max()), float(d.mean())
@@ -68,6 +79,15 @@ def attn_errors(gpu: np.ndarray, ref: np.ndarray):
 
 def rows_of_units(unit_start_tokens: np.ndarray, units) -> np.ndarray:
     return np.concatenate([np.arange(unit_start_tokens[u], unit_start_tokens[u + 1]) for u in units])
+
+
+def last_query_blocks(w, unit_start: np.ndarray, units, rows: int = 128) -> np.ndarray:
+    """Every row of the last `rows`-row query block of each listed unit: the
+    rows with the longest cluster-spanning window, the attention kernel's
+    heaviest work items."""
+    tok = np.minimum(np.asarray(unit_start, np.int64) * w.sub_chunk, w.n_tokens)
+    out = [np.arange(max(tok[u], tok[u + 1] - rows), tok[u + 1]) for u in units]
+    return np.concatenate(out) if out else np.zeros(0, np.int64)
 
 
 def sample_rows(w, unit_start: np.ndarray, n_random: int, seed: int = 1234) -> np.ndarray:
