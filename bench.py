@@ -1,13 +1,16 @@
 #!/usr/bin/env python
 """Benchmark of the Similarity Chunk Rolling sparse-prefill path on GB300.
 
-One step = steps (a)-(d) of the path over one layer of the workload: block
-representatives + fingerprints + anchor clusters, cluster-level selection,
-block-sparse causal attention. Inputs are resident in HBM before timing; they
-are larger than L2 (Q, K, V of the 128K workload are 1.6 GB).
+One step = steps (a)-(d) of the path over one layer of the workload, in the
+order of chunked prefill (Algorithm 2): for every outer chunk, the block
+representatives, fingerprints and anchor clusters of the chunk, then one
+selection and one block-sparse causal attention call per unit (cluster, or
+sub-chunk in the per-sub-chunk mode). The same layer with all units in one
+launch per step is reported as "batched". Inputs are resident in HBM before
+timing; they are larger than L2 (Q, K, V of the 128K workload are 1.6 GB).
 
 Prints one JSON line (rank 0). ``--impl reference`` times the CPU fp64 oracle
-instead, on a bounded sample of the same workload.
+instead, on the same bounded sample of the same workload as the CPU leg.
 """
 
 from __future__ import annotations
@@ -45,12 +48,10 @@ def parse_args():
     ap.add_argument("--mode", choices=["cluster", "subchunk"], default="cluster")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--no-chunk-loop", action="store_true",
-                    help="skip timing the per-outer-chunk loop of range calls alongside")
+    ap.add_argument("--no-cpu-full", action="store_true",
+                    help="skip timing the oracle over every row of the 4K and 32K layers")
     ap.add_argument("--no-baseline-mode", action="store_true",
                     help="skip timing the per-sub-chunk selection mode alongside")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0,
-                    help="target CPU time of the oracle sample")
     ap.add_argument("--paged", type=int, default=0, metavar="P",
                     help="keep K and V in a paged cache of P-token pages (shuffled page order)")
     ap.add_argument("--decode", action="store_true",
@@ -128,27 +129,19 @@ def key_counts(w, unit_start, n_units, sel, cnt, per_subchunk):
     return total
 
 
-def profile_traffic(workload_name: str):
-    """Per-launch DRAM bytes of the attention kernel on this workload from the
-    committed ncu summary (profiles/attn_<workload>_ncu.md), or None when there
-    is none or the kernel source changed since the capture."""
-    summary = os.path.join(PROFILE_DIR, f"attn_{workload_name}_ncu.md")
-    if not os.path.exists(summary):
-        return None
+def profile_counters(workload_name: str) -> dict:
+    """ncu counters of the attention kernel on this workload, from the
+    machine-readable sidecar committed beside its summary
+    (profiles/attn_<workload>_ncu.json). Empty when there is none or when the
+    kernel source changed since the capture (its hash is stored with it)."""
+    path = os.path.join(PROFILE_DIR, f"attn_{workload_name}_ncu.json")
+    if not os.path.exists(path):
+        return {}
     with open(KERNEL_SRC, "rb") as f:
         sha = hashlib.sha256(f.read()).hexdigest()[:16]
-    vals = {}
-    with open(summary) as f:
-        for line in f:
-            if ": " in line and line.strip().startswith("- "):
-                k, v = line.strip()[2:].split(": ", 1)  # keys may hold a colon ("sha256[:16]")
-                vals[k.strip()] = v.strip()
-    if vals.get("attn.cu sha256[:16]") != sha:
-        return None
-    try:
-        return float(vals["traffic bytes per full launch"])
-    except (KeyError, ValueError):
-        return None
+    with open(path) as f:
+        rec = json.load(f)
+    return rec if rec.get("kernel_source_sha16") == sha else {}
 
 
 class ClockSampler:
@@ -213,36 +206,71 @@ class ClockSampler:
 
 # --------------------------------------------------------------------------- oracle timing
 
+# The oracle's row sample: the same seeded rows in the main arm's CPU leg and
+# in the reference arm, so that the two report the same quantity.
+ORACLE_ROWS = 512
+ORACLE_ROW_SEED = 7
+# Workloads the CPU leg also times in full (every row of Eq. 10).
+FULL_ORACLE_WORKLOADS = ("gqa4-4k", "llama8b-32k")
 
-def oracle_sample(w, q, k, v, per_subchunk, cpu_seconds, rows_first=32):
-    """Time the oracle on a bounded sample: steps (a)-(c) over the whole layer,
-    step (d) on a growing set of seeded rows until about cpu_seconds; the
-    throughput is extrapolated from the per-row time to all rows."""
+
+def _cores() -> int:
+    omp = os.environ.get("OMP_NUM_THREADS")
+    if omp:
+        return int(omp)
+    return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+
+
+def oracle_sample(w, q, k, v, per_subchunk, rows=ORACLE_ROWS, seed=ORACLE_ROW_SEED):
+    """One timed run of the oracle on a bounded sample: steps (a)-(c) over the
+    whole layer, Eq. 10 on `rows` seeded rows (all rows when rows >= N). The
+    throughput extrapolates the per-row time of Eq. 10 to every row."""
     import oracle
 
     t0 = time.perf_counter()
     ref = oracle.run_path(w, q, k, v, per_subchunk=per_subchunk)
     t_abc = time.perf_counter() - t0
-    rng = np.random.default_rng(7)
-    n_rows, t_d, done = rows_first, 0.0, 0
-    while True:
-        rows = np.sort(rng.integers(0, w.n_tokens, size=n_rows))
-        t1 = time.perf_counter()
-        oracle.attention_rows(q=q, k=k, v=v, sub_chunk=w.sub_chunk, block_size=w.block_size,
-                              top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
-                              attn_scale=1.0 / np.sqrt(w.head_dim), per_subchunk=per_subchunk,
-                              unit_start=ref["unit_start"], sel=ref["sel"],
-                              sel_count=ref["sel_count"], rows=rows)
-        t_d += time.perf_counter() - t1
-        done += n_rows
-        if t_abc + t_d >= cpu_seconds or done >= w.n_tokens:
-            break
-        n_rows = min(w.n_tokens, max(n_rows, int(n_rows * max(1.5, (cpu_seconds - t_abc) / max(t_d, 1e-3) * 0.6))))
-    t_full = t_abc + t_d / done * w.n_tokens
-    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
-    omp = os.environ.get("OMP_NUM_THREADS")
-    return dict(tokens_per_s=w.n_tokens / t_full, t_full=t_full, t_abc=t_abc, t_d=t_d, rows=done,
-                cores=int(omp) if omp else cores)
+    if rows >= w.n_tokens:
+        sample = np.arange(w.n_tokens, dtype=np.int64)
+    else:
+        sample = np.sort(np.random.default_rng(seed).choice(w.n_tokens, size=rows, replace=False))
+    t1 = time.perf_counter()
+    oracle.attention_rows(q=q, k=k, v=v, sub_chunk=w.sub_chunk, block_size=w.block_size,
+                          top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                          attn_scale=1.0 / np.sqrt(w.head_dim), per_subchunk=per_subchunk,
+                          unit_start=ref["unit_start"], sel=ref["sel"],
+                          sel_count=ref["sel_count"], rows=sample)
+    t_d = time.perf_counter() - t1
+    n = len(sample)
+    t_full = t_abc + t_d / n * w.n_tokens
+    return dict(tokens_per_s=w.n_tokens / t_full, t_full=t_full, t_abc=t_abc, t_d=t_d, t_run=t_abc + t_d,
+                rows=n, extrapolated=n < w.n_tokens, cores=_cores(), ref=ref)
+
+
+def sample_label(w, r) -> str:
+    if not r["extrapolated"]:
+        return (f"the whole layer: steps (a)-(c) and Eq. 10 on all {w.n_tokens} rows "
+                f"({r['t_abc']:.2f} s + {r['t_d']:.2f} s)")
+    return (f"steps (a)-(c) over all {w.n_tokens} tokens ({r['t_abc']:.2f} s) + Eq. 10 on {r['rows']} "
+            f"seeded rows ({r['t_d']:.2f} s); Eq. 10's time per row extrapolated to all {w.n_tokens} rows")
+
+
+def selection_agreement(w, ref, sel, cnt) -> dict:
+    """GPU selection against the oracle's, unit by unit: identical, different
+    at a near-tie (oracle k-th vs (k+1)-th relative gap < 1e-3: both are
+    correct), and different otherwise (a parity failure)."""
+    n = len(ref["sel_count"])
+    match = near = bad = 0
+    for u in range(n):
+        c = int(ref["sel_count"][u])
+        if int(cnt[u]) == c and np.array_equal(sel[u, :c], ref["sel"][u, :c]):
+            match += 1
+        elif ref["gap"][u] < 1e-3:
+            near += 1
+        else:
+            bad += 1
+    return {"selection_match_units": match, "near_tie_units": near, "selection_mismatch_units": bad,
+            "units": n, "near_tie_gap": 1e-3}
 
 
 # --------------------------------------------------------------------------- arms
@@ -256,34 +284,56 @@ def dist_setup(args):
 
 
 def run_reference(args):
+    """The oracle as the reference arm: every step is the same bounded sample
+    as the main arm's CPU leg (steps (a)-(c) over the layer + Eq. 10 on
+    ORACLE_ROWS seeded rows). ms_per_step is the time of what ran; value is
+    the extrapolated whole-layer throughput, labelled as such."""
     world, rank, local = dist_setup(args)
     if rank != 0:
         return 0
     w = workload(args.workload)
     per_sub = args.mode == "subchunk"
     q, k, v = generate_layer(w)
-    times, last = [], None
+    runs = []
     for i in range(args.warmup + args.steps):
-        r = oracle_sample(w, q, k, v, per_sub, cpu_seconds=max(1.0, args.cpu_seconds / 4), rows_first=16)
+        r = oracle_sample(w, q, k, v, per_sub)
+        r.pop("ref")
         if i >= args.warmup:
-            times.append(r["t_full"])
-            last = r
-    t = statistics.mean(times)
-    value = w.n_tokens / t
-    sample = (f"per step: steps (a)-(c) over all {w.n_tokens} tokens ({last['t_abc']:.2f} s) + "
-              f"Eq. 10 on {last['rows']} seeded rows ({last['t_d']:.2f} s), extrapolated per row")
+            runs.append(r)
+    t_full = statistics.mean(r["t_full"] for r in runs)
+    t_run = statistics.mean(r["t_run"] for r in runs)
+    value = w.n_tokens / t_full
+    last = runs[-1]
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
-        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3,
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_run * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
         "config": {"workload": w.name, "n_tokens": w.n_tokens, "mode": args.mode, "theta": w.theta},
+        "extrapolated": last["extrapolated"], "rows_timed": last["rows"], "rows_total": w.n_tokens,
+        "ms_per_step_extrapolated": t_full * 1e3,
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": last["cores"], "kind": "oracle",
-                         "sample": sample},
+                         "sample": "per step: " + sample_label(w, last), "extrapolated": last["extrapolated"],
+                         "rows_timed": last["rows"], "rows_total": w.n_tokens},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
+
+
+def loop_calls(w, mode_sub: bool):
+    """One step of chunked prefill as Algorithm 2 orders it: for every outer
+    chunk, step (a) over the chunk, then one selection and one attention call
+    per unit. A per-sub-chunk unit is one sub-chunk; in SCR mode the calls
+    cover the chunk's clusters (one per chunk when theta admits every
+    sub-chunk and the outer chunk is one cluster long, as in the timed
+    workloads). Returns [(chunk range, [unit ranges])]."""
+    out = []
+    for t0 in range(0, w.n_tokens, w.outer_chunk):
+        t1 = min(w.n_tokens, t0 + w.outer_chunk)
+        units = ([(a, min(t1, a + w.sub_chunk)) for a in range(t0, t1, w.sub_chunk)] if mode_sub else [(t0, t1)])
+        out.append(((t0, t1), units))
+    return out
 
 
 def run_scale(args):
@@ -307,7 +357,6 @@ def run_scale(args):
     q, k, v = generate_layer(w, seed=w.seed + rank)
     dev = [torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)]
     p = S.params_for(w)
-    buf = pkg.allocate(p, mode)
     stream = torch.cuda.current_stream()
     kv = None
     if args.paged:
@@ -329,70 +378,121 @@ def run_scale(args):
         if world > 1:
             torch.distributed.barrier()
 
-    def timed(mode_, steps, warmup, buf_):
-        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(steps)]
-        for _ in range(warmup):
-            pkg.run_path(p, mode_, *dev, buf_)
-        torch.cuda.synchronize()
-        barrier()
-        torch.cuda.synchronize()
-        clocks = ClockSampler(torch.cuda.current_device())
-        clocks.start()
-        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        start.record(stream)
-        for i in range(steps):
-            e = ev[i]
-            e[0].record(stream)
-            if kv is not None:
+    def build(buf_, t0, t1, whole):
+        if kv is not None:
+            if whole:
                 S.scale_build_reps_paged(p, dev[0], kv, buf_.reps, buf_.fingerprints, buf_.unit_start,
                                          buf_.n_units, buf_.ws, stream)
             else:
-                S.scale_build_reps(p, dev[0], dev[1], buf_.reps, buf_.fingerprints, buf_.unit_start,
-                                   buf_.n_units, buf_.ws, stream)
-            e[1].record(stream)
-            if kv is not None and w.block_size == 1:
-                S.scale_select_tokens_paged(p, mode_, 0, w.n_tokens, kv, buf_.fingerprints, buf_.unit_start,
-                                            buf_.n_units, buf_.sel_blocks, buf_.sel_count, None, buf_.ws,
-                                            stream)
-            else:
-                S.select(p, mode_, 0, w.n_tokens, dev[1], buf_, stream)
-            e[2].record(stream)
-            if kv is not None:
-                S.scale_sparse_prefill_paged(p, mode_, 0, w.n_tokens, dev[0], kv, buf_.unit_start,
-                                             buf_.n_units, buf_.sel_blocks, buf_.sel_count, buf_.out,
-                                             buf_.ws, stream)
-            else:
-                S.scale_sparse_prefill(p, mode_, 0, w.n_tokens, *dev, buf_.unit_start, buf_.n_units,
-                                       buf_.sel_blocks, buf_.sel_count, buf_.out, buf_.ws, stream)
-            e[3].record(stream)
+                S.scale_build_reps_range_paged(p, t0, t1, dev[0], kv, buf_.reps, buf_.fingerprints,
+                                               buf_.unit_start, buf_.n_units, buf_.ws, stream)
+        elif whole:
+            S.scale_build_reps(p, dev[0], dev[1], buf_.reps, buf_.fingerprints, buf_.unit_start,
+                               buf_.n_units, buf_.ws, stream)
+        else:
+            S.scale_build_reps_range(p, t0, t1, dev[0], dev[1], buf_.reps, buf_.fingerprints,
+                                     buf_.unit_start, buf_.n_units, buf_.ws, stream)
+
+    def select(mode_, buf_, t0, t1):
+        if kv is not None and w.block_size == 1:
+            S.scale_select_tokens_paged(p, mode_, t0, t1, kv, buf_.fingerprints, buf_.unit_start,
+                                        buf_.n_units, buf_.sel_blocks, buf_.sel_count, None, buf_.ws, stream)
+        else:
+            S.select(p, mode_, t0, t1, dev[1], buf_, stream)
+
+    def attend(mode_, buf_, t0, t1):
+        if kv is not None:
+            S.scale_sparse_prefill_paged(p, mode_, t0, t1, dev[0], kv, buf_.unit_start, buf_.n_units,
+                                         buf_.sel_blocks, buf_.sel_count, buf_.out, buf_.ws, stream)
+        else:
+            S.scale_sparse_prefill(p, mode_, t0, t1, *dev, buf_.unit_start, buf_.n_units,
+                                   buf_.sel_blocks, buf_.sel_count, buf_.out, buf_.ws, stream)
+
+    def step_plan(mode_, batched):
+        """[(build range, [(select/attend range)])] of one step."""
+        if batched:
+            return [((0, w.n_tokens), [(0, w.n_tokens)])]
+        return loop_calls(w, mode_ == S.SCALE_MODE_PER_SUBCHUNK)
+
+    def timed(mode_, batched, steps, warmup, buf_, sample_clocks=False):
+        """Time `steps` steps (CUDA events on the launch stream): the whole step,
+        and the three stages summed over their calls within it."""
+        plan = step_plan(mode_, batched)
+        n_calls = sum(len(u) for _, u in plan)
+
+        def one(ev):
+            def rec(stage, j):
+                if ev is not None:
+                    ev[stage][j].record(stream)
+
+            j = 0
+            for (c0, c1), units in plan:
+                for i, (t0, t1) in enumerate(units):
+                    rec(0, j)
+                    if i == 0:
+                        build(buf_, c0, c1, batched)
+                    rec(1, j)
+                    select(mode_, buf_, t0, t1)
+                    rec(2, j)
+                    attend(mode_, buf_, t0, t1)
+                    rec(3, j)
+                    j += 1
+
+        for _ in range(warmup):
+            one(None)
+        torch.cuda.synchronize()
+        barrier()
+        torch.cuda.synchronize()
+        evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(n_calls)] for _ in range(4)]
+               for _ in range(steps)]
+        clocks = ClockSampler(torch.cuda.current_device()) if sample_clocks else None
+        if clocks:
+            clocks.start()
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        for i in range(steps):
+            one(evs[i])
         end.record(stream)
         torch.cuda.synchronize()
-        clk = clocks.stop()
+        clk = clocks.stop() if clocks else None
         barrier()
         total = start.elapsed_time(end) / steps
-        stages = [statistics.mean(x[j].elapsed_time(x[j + 1]) for x in ev) for j in range(3)]
+        # stage sums per step (a unit after its chunk's first has no build)
+        stages = [statistics.mean(sum(e[jj][c].elapsed_time(e[jj + 1][c]) for c in range(n_calls)) for e in evs)
+                  for jj in range(3)]
         st = S.scale_get_device_status(buf_.ws)
         if st != S.SCALE_OK:
             raise RuntimeError(f"device status {st}: {S.status_string(st)}")
-        return total, stages, clk
+        return {"ms_per_step": total, "tokens_per_s": w.n_tokens / (total / 1e3),
+                "stages_ms": {"build_reps": stages[0], "select": stages[1], "sparse_attention": stages[2]},
+                "build_calls": len(plan), "select_attend_calls": n_calls,
+                "gpu_launches": launches(w, n_calls, len(plan))["total"]}, clk
 
-    ms, stages, clk = timed(mode, args.steps, args.warmup, buf)
+    def unit_stats(mode_, buf_):
+        sub = mode_ == S.SCALE_MODE_PER_SUBCHUNK
+        n = w.n_subchunks if sub else int(buf_.n_units.item())
+        us = buf_.unit_start.cpu().numpy()
+        sel = buf_.sel_blocks.cpu().numpy()
+        cnt = buf_.sel_count.cpu().numpy()
+        keys = key_counts(w, us, n, sel, cnt, sub)
+        _, calls = S.scale_retrieval_calls(p, mode_, None if sub else us[: n + 1], n)
+        return n, calls, 4.0 * w.head_dim * w.num_q_heads * keys, sel[:n], cnt[:n]
+
+    buf = pkg.allocate(p, mode)
+    # headline: the chunked-prefill loop of Algorithm 2
+    head, clk = timed(mode, False, args.steps, args.warmup, buf, sample_clocks=True)
+    ms = head["ms_per_step"]
     if world > 1:
         t = torch.tensor([ms], device="cuda")
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms = float(t.item())
-
-    n_units = w.n_subchunks if per_sub else int(buf.n_units.item())
-    us = buf.unit_start.cpu().numpy()
-    sel = buf.sel_blocks.cpu().numpy()
-    cnt = buf.sel_count.cpu().numpy()
-    keys = key_counts(w, us, n_units, sel, cnt, per_sub)
-    flops = 4.0 * w.head_dim * w.num_q_heads * keys
+    n_units, calls, flops, sel_gpu, cnt_gpu = unit_stats(mode, buf)
     peaks = load_peaks()
-    attn_s = stages[2] / 1e3
-    achieved = flops / attn_s / 1e12
-    _, calls = S.scale_retrieval_calls(p, mode, us[: n_units + 1] if not per_sub else None, n_units)
-
+    attn_ms = head["stages_ms"]["sparse_attention"]
+    n_attn = head["select_attend_calls"]
+    achieved = flops / (attn_ms / 1e3) / 1e12
+    prof = profile_counters(w.name) if kv is None else {}
+    mode_name = "subchunk" if per_sub else "cluster"
     line = {
         "metric": METRIC,
         "value": world * w.n_tokens / (ms / 1e3),
@@ -409,82 +509,59 @@ def run_scale(args):
         "data": "synthetic",
         "config": {"workload": w.name, "n_tokens": w.n_tokens, "q_heads": w.num_q_heads,
                    "kv_heads": w.num_kv_heads, "head_dim": w.head_dim, "sub_chunk": w.sub_chunk,
-                   "max_cluster_subchunks": w.max_cluster_subchunks, "block_size": w.block_size,
-                   "top_k": w.top_k, "n_sink": w.n_sink, "n_local": w.n_local, "theta": w.theta,
-                   "mode": args.mode, "parallelism": f"independent layers x{world}",
+                   "outer_chunk": w.outer_chunk, "max_cluster_subchunks": w.max_cluster_subchunks,
+                   "block_size": w.block_size, "top_k": w.top_k, "n_sink": w.n_sink, "n_local": w.n_local,
+                   "theta": w.theta, "mode": mode_name, "parallelism": f"independent layers x{world}",
+                   "loop": ("Algorithm 2: per outer chunk scale_build_reps_range, then one scale_select and "
+                            "one scale_sparse_prefill per unit (" +
+                            ("sub-chunk" if per_sub else "cluster; one per outer chunk at theta = -1") + ")"),
                    "kv_layout": f"paged, {args.paged}-token pages" if args.paged else "contiguous",
                    "l2": "inputs larger than L2 (Q+K+V %.2f GB)" % ((q.nbytes + k.nbytes + v.nbytes) / 1e9)},
-        "stages_ms": {"build_reps": stages[0], "select": stages[1], "sparse_attention": stages[2]},
+        "stages_ms": head["stages_ms"],
+        "calls_per_step": {"build_reps_range": head["build_calls"], "select": n_attn, "sparse_prefill": n_attn},
         "retrieval_calls": calls,
         "units": n_units,
         "roofline": {"bound": "tensor", "kernel": "k_sparse_attn", "achieved": achieved,
-                     "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
-                     "frac": achieved / peaks["bf16_sustained"],
-                     "frac_of_burst": achieved / peaks["bf16"],
-                     "peak_source": f"bf16 sustained, of {peaks['source']}",
-                     "algorithmic_flops_per_launch": flops, "traffic": profile_traffic(w.name)},
-        "gpu_launches": args.steps * launches(w)["total"],
+                     "peak": peaks["bf16"], "unit": "TFLOP/s", "frac": achieved / peaks["bf16"],
+                     "peak_source": f"bf16 burst, of {peaks['source']}",
+                     "frac_of_sustained": achieved / peaks["bf16_sustained"],
+                     "launches_per_step": n_attn,
+                     "algorithmic_flops_per_launch": flops / n_attn,
+                     "ms_per_launch": attn_ms / n_attn,
+                     "traffic": prof.get("traffic_bytes_per_launch"),
+                     "tensor_pipe_active_pct": prof.get("tensor_pipe_active_pct"),
+                     "counters_from": prof.get("summary")},
+        "gpu_launches": args.steps * head["gpu_launches"],
         "clocks": clk,
     }
+
+    if rank == 0:
+        bat, _ = timed(mode, True, max(3, args.steps // 2), 2, buf)
+        line["batched"] = dict(bat, loop="whole sequence: scale_build_reps, scale_select, scale_sparse_prefill "
+                                         "(all units of the layer in one launch each)")
 
     if not args.no_baseline_mode and rank == 0:
         other = S.SCALE_MODE_PER_SUBCHUNK if not per_sub else S.SCALE_MODE_PER_CLUSTER
         buf2 = pkg.allocate(p, other)
-        ms2, st2, _ = timed(other, max(3, args.steps // 2), 2, buf2)
-        n2 = w.n_subchunks if other == S.SCALE_MODE_PER_SUBCHUNK else int(buf2.n_units.item())
-        us2 = buf2.unit_start.cpu().numpy()
-        _, calls2 = S.scale_retrieval_calls(
-            p, other, us2[: n2 + 1] if other == S.SCALE_MODE_PER_CLUSTER else None, n2)
-        line["other_mode"] = {"mode": "subchunk" if other == S.SCALE_MODE_PER_SUBCHUNK else "cluster",
-                              "ms_per_step": ms2, "tokens_per_s": w.n_tokens / (ms2 / 1e3),
-                              "stages_ms": {"build_reps": st2[0], "select": st2[1], "sparse_attention": st2[2]},
-                              "retrieval_calls": calls2, "units": n2}
+        o_loop, _ = timed(other, False, max(3, args.steps // 2), 2, buf2)
+        o_bat, _ = timed(other, True, max(3, args.steps // 2), 2, buf2)
+        n2, calls2, flops2, _, _ = unit_stats(other, buf2)
+        other_name = "subchunk" if other == S.SCALE_MODE_PER_SUBCHUNK else "cluster"
+        line["other_mode"] = dict(o_loop, mode=other_name, retrieval_calls=calls2, units=n2,
+                                  attn_tflops=flops2 / (o_loop["stages_ms"]["sparse_attention"] / 1e3) / 1e12,
+                                  batched=o_bat)
+        scr, sub = (head, o_loop) if not per_sub else (o_loop, head)
+        scr_b, sub_b = (line["batched"], o_bat) if not per_sub else (o_bat, line["batched"])
+        f_scr, f_sub = (flops, flops2) if not per_sub else (flops2, flops)
+        line["scr_over_subchunk"] = scr["ms_per_step"] / sub["ms_per_step"]
+        line["scr_over_subchunk_batched"] = scr_b["ms_per_step"] / sub_b["ms_per_step"]
+        line["attn_flops_ratio"] = f_scr / f_sub
+        line["retrieval"] = {
+            "cluster": {"calls": calls if not per_sub else calls2,
+                        "select_ms": scr["stages_ms"]["select"]},
+            "subchunk": {"calls": calls2 if not per_sub else calls,
+                         "select_ms": sub["stages_ms"]["select"]}}
         del buf2
-
-    if not args.no_chunk_loop and rank == 0:
-        # Chunked prefill as Algorithm 2 orders it: per outer chunk, step (a)
-        # over the chunk's range, then its selection and attention.
-        chunks = [(t0, min(w.n_tokens, t0 + w.outer_chunk)) for t0 in range(0, w.n_tokens, w.outer_chunk)]
-
-        def chunk_step():
-            for t0, t1 in chunks:
-                if kv is not None:
-                    S.scale_build_reps_range_paged(p, t0, t1, dev[0], kv, buf.reps, buf.fingerprints,
-                                                   buf.unit_start, buf.n_units, buf.ws, stream)
-                    if w.block_size == 1:
-                        S.scale_select_tokens_paged(p, mode, t0, t1, kv, buf.fingerprints, buf.unit_start,
-                                                    buf.n_units, buf.sel_blocks, buf.sel_count, None, buf.ws,
-                                                    stream)
-                    else:
-                        S.select(p, mode, t0, t1, None, buf, stream)
-                    S.scale_sparse_prefill_paged(p, mode, t0, t1, dev[0], kv, buf.unit_start, buf.n_units,
-                                                 buf.sel_blocks, buf.sel_count, buf.out, buf.ws, stream)
-                else:
-                    S.scale_build_reps_range(p, t0, t1, dev[0], dev[1], buf.reps, buf.fingerprints,
-                                             buf.unit_start, buf.n_units, buf.ws, stream)
-                    S.select(p, mode, t0, t1, dev[1], buf, stream)
-                    S.scale_sparse_prefill(p, mode, t0, t1, *dev, buf.unit_start, buf.n_units,
-                                           buf.sel_blocks, buf.sel_count, buf.out, buf.ws, stream)
-
-        for _ in range(2):
-            chunk_step()
-        torch.cuda.synchronize()
-        c_steps = max(3, args.steps // 2)
-        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        start.record(stream)
-        for _ in range(c_steps):
-            chunk_step()
-        end.record(stream)
-        torch.cuda.synchronize()
-        st = S.scale_get_device_status(buf.ws)
-        if st != S.SCALE_OK:
-            raise RuntimeError(f"device status {st}: {S.status_string(st)}")
-        ms_c = start.elapsed_time(end) / c_steps
-        line["chunk_loop"] = {"ms_per_step": ms_c, "tokens_per_s": w.n_tokens / (ms_c / 1e3),
-                              "outer_chunks": len(chunks),
-                              "calls_per_step": 3 * len(chunks),
-                              "kernel_launches_per_step": launches(w, len(chunks), len(chunks))["total"],
-                              "loop": "per outer chunk: scale_build_reps_range, select, scale_sparse_prefill"}
 
     if not args.no_e2e:
         qh, kh, vh = (torch.from_numpy(x).pin_memory() for x in (q, k, v))
@@ -510,15 +587,26 @@ def run_scale(args):
                        "d2h_bytes_per_step": int(q.nbytes), "ms_per_step": t_e2e * 1e3,
                        "ms_min": min(per_call) * 1e3, "ms_median": statistics.median(per_call) * 1e3,
                        "host_link_gbs": link,
-                       "api": "scale_prefill_host (pinned host buffers)"}
+                       "api": "scale_prefill_host (pinned host buffers; pieces of outer chunks, copies "
+                              "overlapped with the compute)"}
         del arena
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        r = oracle_sample(w, q, k, v, per_sub, args.cpu_seconds)
+        r = oracle_sample(w, q, k, v, per_sub)
+        line.update(selection_agreement(w, r["ref"], sel_gpu, cnt_gpu))
         line["cpu_baseline"] = {
             "value": r["tokens_per_s"], "unit": "tokens/s", "cores": r["cores"], "kind": "oracle",
-            "sample": (f"steps (a)-(c) over all {w.n_tokens} tokens ({r['t_abc']:.2f} s) + Eq. 10 on "
-                       f"{r['rows']} seeded rows ({r['t_d']:.2f} s), time per row extrapolated to all rows")}
+            "sample": sample_label(w, r), "extrapolated": r["extrapolated"], "rows_timed": r["rows"],
+            "rows_total": w.n_tokens, "ms_run": r["t_run"] * 1e3}
+        if not args.no_cpu_full and w.name == DEFAULT_WORKLOAD:
+            full = {}
+            for name in FULL_ORACLE_WORKLOADS:
+                wf = workload(name)
+                qf, kf, vf = generate_layer(wf)
+                rf = oracle_sample(wf, qf, kf, vf, per_sub, rows=wf.n_tokens)
+                full[name] = {"tokens_per_s": rf["tokens_per_s"], "s": rf["t_full"], "extrapolated": False,
+                              "sample": sample_label(wf, rf)}
+            line["cpu_baseline"]["full_layers"] = full
 
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -760,26 +848,26 @@ def run_stack(args):
         q, k, v = generate_layer(w, layer=l, seed=w.seed + l + 1000 * rank)
         layers.append([torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)])
         del q, k, v
-    chunks = [(t0, min(w.n_tokens, t0 + w.outer_chunk)) for t0 in range(0, w.n_tokens, w.outer_chunk)]
-
     def measure(mode, steps, warmup):
         bufs = [pkg.allocate(p, mode) for _ in layers]
-        n_attn = len(chunks) * len(layers)
+        plan = loop_calls(w, mode == S.SCALE_MODE_PER_SUBCHUNK)
+        n_attn = sum(len(u) for _, u in plan) * len(layers)
 
         def step(ev=None):
             i = 0
-            for t0, t1 in chunks:
+            for (c0, c1), units in plan:
                 for dev, b in zip(layers, bufs):
-                    S.scale_build_reps_range(p, t0, t1, dev[0], dev[1], b.reps, b.fingerprints, b.unit_start,
+                    S.scale_build_reps_range(p, c0, c1, dev[0], dev[1], b.reps, b.fingerprints, b.unit_start,
                                              b.n_units, b.ws, stream)
-                    S.select(p, mode, t0, t1, dev[1], b, stream)
-                    if ev is not None:
-                        ev[i][0].record(stream)
-                    S.scale_sparse_prefill(p, mode, t0, t1, *dev, b.unit_start, b.n_units, b.sel_blocks,
-                                           b.sel_count, b.out, b.ws, stream)
-                    if ev is not None:
-                        ev[i][1].record(stream)
-                    i += 1
+                    for t0, t1 in units:
+                        S.select(p, mode, t0, t1, dev[1], b, stream)
+                        if ev is not None:
+                            ev[i][0].record(stream)
+                        S.scale_sparse_prefill(p, mode, t0, t1, *dev, b.unit_start, b.n_units, b.sel_blocks,
+                                               b.sel_count, b.out, b.ws, stream)
+                        if ev is not None:
+                            ev[i][1].record(stream)
+                        i += 1
 
         for _ in range(warmup):
             step()
@@ -813,10 +901,11 @@ def run_stack(args):
             units += n
             calls += S.scale_retrieval_calls(p, mode, None if per_sub else us[: n + 1], n)[1]
         del bufs
-        return ms, attn_ms, clk, 4.0 * w.head_dim * w.num_q_heads * keys, calls, units
+        launch_count = w.layers * launches(w, n_attn // w.layers, len(plan))["total"]
+        return ms, attn_ms, clk, 4.0 * w.head_dim * w.num_q_heads * keys, calls, units, launch_count, n_attn
 
     mode = S.SCALE_MODE_PER_SUBCHUNK if args.mode == "subchunk" else S.SCALE_MODE_PER_CLUSTER
-    ms, attn_ms, clk, flops, calls, units = measure(mode, args.steps, args.warmup)
+    ms, attn_ms, clk, flops, calls, units, n_launch, n_attn = measure(mode, args.steps, args.warmup)
     if world > 1:
         t = torch.tensor([ms], device="cuda")
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
@@ -829,25 +918,31 @@ def run_stack(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": w.name, "n_tokens": w.n_tokens, "layers": w.layers, "mode": args.mode,
-                   "outer_chunk": w.outer_chunk, "loop": "chunk-major: every layer per outer chunk",
+                   "outer_chunk": w.outer_chunk,
+                   "loop": ("Algorithm 2, chunk-major: per outer chunk and layer scale_build_reps_range, then one "
+                            "scale_select and one scale_sparse_prefill per unit"),
                    "parallelism": f"independent stacks x{world}", "l2": "inputs larger than L2"},
         "stages_ms": {"sparse_attention_total": attn_ms, "other": ms - attn_ms},
         "retrieval_calls": calls, "units": units,
         "roofline": {"bound": "tensor", "kernel": "k_sparse_attn", "achieved": achieved,
-                     "peak": peaks["bf16_sustained"], "unit": "TFLOP/s",
-                     "frac": achieved / peaks["bf16_sustained"], "frac_of_burst": achieved / peaks["bf16"],
-                     "peak_source": f"bf16 sustained, of {peaks['source']}",
-                     "algorithmic_flops_per_step": flops, "traffic": None},
-        "gpu_launches": args.steps * w.layers * launches(w, len(chunks), len(chunks))["total"],
+                     "peak": peaks["bf16"], "unit": "TFLOP/s", "frac": achieved / peaks["bf16"],
+                     "peak_source": f"bf16 burst, of {peaks['source']}",
+                     "frac_of_sustained": achieved / peaks["bf16_sustained"],
+                     "launches_per_step": n_attn, "algorithmic_flops_per_launch": flops / n_attn,
+                     "traffic": None},
+        "gpu_launches": args.steps * n_launch,
         "clocks": clk,
     }
     if not args.no_baseline_mode and rank == 0:
         other = S.SCALE_MODE_PER_SUBCHUNK if mode == S.SCALE_MODE_PER_CLUSTER else S.SCALE_MODE_PER_CLUSTER
-        ms2, attn2, _, flops2, calls2, units2 = measure(other, max(2, args.steps // 2), 1)
+        ms2, attn2, _, flops2, calls2, units2, _, _ = measure(other, max(2, args.steps // 2), 1)
         line["other_mode"] = {"mode": "subchunk" if other == S.SCALE_MODE_PER_SUBCHUNK else "cluster",
                               "ms_per_step": ms2, "tokens_per_s": w.n_tokens / (ms2 / 1e3),
                               "sparse_attention_ms": attn2, "retrieval_calls": calls2, "units": units2,
                               "attn_tflops": flops2 / (attn2 / 1e3) / 1e12}
+        per_sub_first = mode == S.SCALE_MODE_PER_SUBCHUNK
+        line["scr_over_subchunk"] = (ms2 / ms) if per_sub_first else (ms / ms2)
+        line["attn_flops_ratio"] = (flops2 / flops) if per_sub_first else (flops / flops2)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -1,10 +1,15 @@
-"""CPU checks of bench.py's bookkeeping: the per-launch DRAM traffic is read
-from the committed ncu summary of the same workload only while the kernel
-source is unchanged, and the launch counts follow the path's kernels."""
+"""CPU checks of bench.py's bookkeeping: the attention kernel's ncu counters
+are read from the committed sidecar of the same workload only while the
+kernel source is unchanged, the launch counts follow the path's kernels, the
+Algorithm 2 loop issues one selection and attention call per unit, and the
+selection agreement counts near-ties apart from mismatches."""
 
 import hashlib
+import json
 import os
 import sys
+
+import numpy as np
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 sys.path.insert(0, ROOT)
@@ -13,18 +18,51 @@ import bench  # noqa: E402
 from synth import workload  # noqa: E402
 
 
-def test_profile_traffic_follows_the_kernel_source(tmp_path, monkeypatch):
+def test_profile_counters_follow_the_kernel_source(tmp_path, monkeypatch):
     src = tmp_path / "attn.cu"
     src.write_bytes(b"// kernel v1\n")
     sha = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
-    summary = tmp_path / "attn_wl-a_ncu.md"
-    summary.write_text(f"# title\n\n- attn.cu sha256[:16]: {sha}\n- traffic bytes per full launch: 12345\n")
+    (tmp_path / "attn_wl-a_ncu.json").write_text(json.dumps(
+        {"kernel_source_sha16": sha, "traffic_bytes_per_launch": 12345, "tensor_pipe_active_pct": 70.0}))
     monkeypatch.setattr(bench, "KERNEL_SRC", str(src))
     monkeypatch.setattr(bench, "PROFILE_DIR", str(tmp_path))
-    assert bench.profile_traffic("wl-a") == 12345.0
-    assert bench.profile_traffic("wl-b") is None  # no capture of that workload
+    assert bench.profile_counters("wl-a")["traffic_bytes_per_launch"] == 12345
+    assert bench.profile_counters("wl-b") == {}  # no capture of that workload
     src.write_bytes(b"// kernel v2\n")  # changed since the capture
-    assert bench.profile_traffic("wl-a") is None
+    assert bench.profile_counters("wl-a") == {}
+
+
+def test_committed_sidecars_are_valid_json():
+    d = os.path.join(ROOT, "profiles")
+    for name in os.listdir(d):
+        if name.endswith(".json"):
+            with open(os.path.join(d, name)) as f:
+                rec = json.load(f)
+            assert len(rec["kernel_source_sha16"]) == 16
+
+
+def test_algorithm2_loop_calls():
+    w = workload("llama8b-128k")
+    scr = bench.loop_calls(w, False)
+    assert len(scr) == 8 and all(len(u) == 1 for _, u in scr)  # one cluster per outer chunk
+    assert scr[0] == ((0, 16384), [(0, 16384)])
+    sub = bench.loop_calls(w, True)
+    assert len(sub) == 8 and sum(len(u) for _, u in sub) == 64  # one call per sub-chunk
+    assert sub[1][1][0] == (16384, 18432)
+    ragged = bench.loop_calls(workload("gqa4-4k", n_tokens=3000), True)
+    assert ragged[-1][1][-1] == (2816, 3000)  # last sub-chunk ends at N
+
+
+def test_selection_agreement_counts():
+    w = workload("gqa4-4k")
+    ref = {"sel": np.array([[1, 2], [3, 4], [5, 6]]), "sel_count": np.array([2, 2, 2]),
+           "gap": np.array([0.5, 1e-4, 0.5])}
+    gpu = np.array([[1, 2], [3, 7], [5, 6]])
+    a = bench.selection_agreement(w, ref, gpu, np.array([2, 2, 2]))
+    assert (a["selection_match_units"], a["near_tie_units"], a["selection_mismatch_units"]) == (2, 1, 0)
+    gpu[2, 1] = 9
+    a = bench.selection_agreement(w, ref, gpu, np.array([2, 2, 2]))
+    assert a["selection_mismatch_units"] == 1
 
 
 def test_launch_counts():
