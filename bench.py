@@ -621,7 +621,7 @@ SWEEP_SMAX = (2, 4, 8)
 
 
 def cosine_stats(fp: np.ndarray) -> dict:
-    """Distribution of cos(v_i, v_{i+1}) over consecutive sub-chunks (the paper's Table 1 format)."""
+    """Distribution of cos(v_i, v_{i+1}) over consecutive sub-chunks (the paper's Table 2 format)."""
     vt = fp / np.linalg.norm(fp, axis=1, keepdims=True)
     c = np.sum(vt[1:] * vt[:-1], axis=1)
     return {"mean": float(c.mean()), "min": float(c.min()), "max": float(c.max()),

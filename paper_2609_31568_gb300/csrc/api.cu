@@ -324,7 +324,7 @@ int scale_select(const scale_params_t* p, int32_t mode, int64_t tok_begin, int64
     if (tok_begin == tok_end) return SCALE_OK;
     return cuda_status(launch_select(d, mode, tok_begin, tok_end, reps, fingerprints, unit_start,
                                      n_units, sel_blocks, sel_count, sel_scores,
-                                     static_cast<uint8_t*>(ws), stream));
+                                     static_cast<uint8_t*>(ws), g_timeout_ns.load(), stream));
 }
 
 static int select_tokens_impl(const Derived& d, int32_t mode, int64_t tok_begin, int64_t tok_end,

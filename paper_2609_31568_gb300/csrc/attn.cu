@@ -324,7 +324,6 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 const int st = t & 1;
                 if (!mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t ks = k_base + st * kTileBytes;
                 for (int qt = 0; qt < 2; ++qt) {
                     if (t > 0) {
                         if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }

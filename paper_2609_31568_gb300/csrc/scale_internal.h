@@ -164,7 +164,7 @@ int outer_chunks(const Derived& d);
 cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
                           const float* reps, const float* fingerprints, const int32_t* unit_start,
                           const int32_t* n_units, int32_t* sel_blocks, int32_t* sel_count,
-                          float* sel_scores, uint8_t* ws, cudaStream_t st);
+                          float* sel_scores, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
                                   const void* q, const void* k, const void* v, const KvPaging& pg,
                                   const int32_t* unit_start, const int32_t* n_units,

@@ -2,7 +2,9 @@
 // retrieval with head soft-voting (Eq. 9, Sec. V-A3 "Selection function
 // instantiation") over block representative keys, then a deterministic top-k.
 //
-//   k_logits  z[u][h][b] = sigma * v_a(u)^(h) . r_b^(h/g)   (fp32 GEMM tile per KV head)
+//   k_logits  z[u][h][b] = sigma * v_a(u)^(h) . r_b^(h/g)   (tcgen05 MMA per KV head:
+//             128 (unit, head) rows x 128 blocks; both fp32 operands split
+//             into three bf16 parts, six part products accumulated in fp32)
 //   k_stats   per (u, h): max_b z and 1 / sum_b exp(z - max) over the candidates
 //   k_vote    score[u][b] = sum_h exp(z[u][h][b] - max) / sum   (heads in order)
 //   k_topk    up to 4096 candidates a bitonic sort of (score, -b) keys in
@@ -13,16 +15,15 @@
 //
 // Candidates of unit u are the blocks with a token in [n_sink, W_u),
 // W_u = max(0, s_u - n_local): the contiguous range [b_lo, b_hi(u)).
+#include <cuda_bf16.h>
+
 #include <cmath>
 
+#include "ptx_sm103.cuh"
 #include "scale_internal.h"
 
 namespace scale {
 namespace {
-
-constexpr int kLogitUnitRows = 32;  // rows (unit, head) per logits tile
-constexpr int kLogitBlocks = 64;    // blocks per logits tile
-constexpr int kLogitThreads = 256;
 
 struct SelArgs {
     Units ut;
@@ -32,6 +33,8 @@ struct SelArgs {
     int B, k, n_sink, n_local;
     float sigma;
     const int32_t* gate;  // nullable: the top-k runs only when *gate != 0
+    int32_t* status;      // device status word (bounded waits of k_logits)
+    uint64_t timeout_ns;
 };
 
 __device__ __forceinline__ void cand_range(const SelArgs& a, int64_t s, int64_t* lo, int64_t* hi)
@@ -43,75 +46,172 @@ __device__ __forceinline__ void cand_range(const SelArgs& a, int64_t s, int64_t*
     if (*hi < *lo) *hi = *lo;
 }
 
-// Grid: (unit tiles, block tiles, KV heads). Rows of the A tile are
-// (unit, query head of this KV head) pairs.
-__global__ void __launch_bounds__(kLogitThreads) k_logits(SelArgs a,
-                                                          const float* __restrict__ fp,
+// Tensor-core logits. Grid: (unit tiles of 128 / g units, 128-block tiles,
+// KV heads j). Rows of the A operand are the (unit, query head of KV head j)
+// pairs of the tile (row ul * g + hl: head j g + hl of unit u0 + ul, the
+// anchor's fingerprint slice), columns of B are the representatives of blocks
+// [b0, b0 + 128) of KV head j. Both are fp32; every value x is split into
+// three bf16 parts x1 + x2 + x3 = x exactly (x1 = bf16(x), x2 = bf16(x - x1),
+// x3 = x - x1 - x2), written by the threads straight into the 128-byte-
+// swizzled K-major layout of the MMA. The six part products a_i b_j with
+// i + j <= 4 are exact in fp32 and are accumulated in fp32 in TMEM; the three
+// dropped ones are below 2^-24 of |a| |b|. Only candidate blocks of each row's
+// unit are written, as before.
+constexpr int kLtThreads = 256;
+constexpr uint32_t kLtPart = 128 * 128 * 2;   // one bf16 part: 128 rows x 128 columns
+constexpr uint32_t kLtHalf = kLtPart / 2;     // one 64-column half
+constexpr uint32_t kLtSmem = 6 * kLtPart + 1024;
+static_assert(kLtSmem <= 227 * 1024, "logits shared memory");
+
+__device__ __forceinline__ void split_bf16x3(float x, __nv_bfloat16& p1, __nv_bfloat16& p2, __nv_bfloat16& p3)
+{
+    p1 = __float2bfloat16_rn(x);
+    const float r1 = x - __bfloat162float(p1);
+    p2 = __float2bfloat16_rn(r1);
+    p3 = __float2bfloat16_rn(r1 - __bfloat162float(p2));
+}
+
+// Four consecutive fp32 values of row r, columns [c, c + 4), into the three
+// bf16 parts at `base` (part s at base + s * kLtPart): 8 bytes per part, at
+// the 128-byte-swizzled K-major position of (r, c).
+__device__ __forceinline__ void put_split4(uint8_t* base, int r, int c, float4 v)
+{
+    __nv_bfloat16 p[3][4];
+    split_bf16x3(v.x, p[0][0], p[1][0], p[2][0]);
+    split_bf16x3(v.y, p[0][1], p[1][1], p[2][1]);
+    split_bf16x3(v.z, p[0][2], p[1][2], p[2][2]);
+    split_bf16x3(v.w, p[0][3], p[1][3], p[2][3]);
+    const int hf = c >> 6, cc = c & 63;  // half, column in the half
+    const uint32_t off = hf * kLtHalf + (r >> 3) * 1024 + (r & 7) * 128 + ((((cc >> 3) ^ (r & 7))) << 4) +
+                         (cc & 7) * 2;
+#pragma unroll
+    for (int s = 0; s < 3; ++s) {
+        uint2 w;
+        w.x = static_cast<uint32_t>(__bfloat16_as_ushort(p[s][0])) |
+              (static_cast<uint32_t>(__bfloat16_as_ushort(p[s][1])) << 16);
+        w.y = static_cast<uint32_t>(__bfloat16_as_ushort(p[s][2])) |
+              (static_cast<uint32_t>(__bfloat16_as_ushort(p[s][3])) << 16);
+        *reinterpret_cast<uint2*>(base + s * kLtPart + off) = w;
+    }
+}
+
+__global__ void __launch_bounds__(kLtThreads, 1) k_logits(SelArgs a, const float* __restrict__ fp,
                                                           const float* __restrict__ reps,
                                                           float* __restrict__ logits)
 {
-    extern __shared__ float sm[];
-    float* As = sm;                                    // [rows][128]
-    float* Bs = sm + kLogitUnitRows * kHeadDim;        // [64][129]
-    const int units_per_tile = kLogitUnitRows / a.g;
-    const int rows = units_per_tile * a.g;
+    using namespace scale_ptx;
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint64_t d_full;
+    __shared__ uint32_t tmem_slot;
+    __shared__ int64_t s_lo[128], s_hi[128];
+    __shared__ int s_anchor[128];
+    __shared__ int any;
+    const int U = 128 / a.g;  // units per tile
     const int u_first = unit_lower_bound(a.ut, a.sc_begin);
     const int u_end = unit_lower_bound(a.ut, a.sc_end);
-    const int u0 = u_first + blockIdx.x * units_per_tile;
+    const int u0 = u_first + static_cast<int>(blockIdx.x) * U;
     if (u0 >= u_end) return;
+    const int n_u = (u_end - u0 < U) ? u_end - u0 : U;
+    const int rows = n_u * a.g;
     const int j = blockIdx.z;
-    const int64_t b0 = static_cast<int64_t>(blockIdx.y) * kLogitBlocks;
+    const int64_t b0 = static_cast<int64_t>(blockIdx.y) * 128;
     const int D = a.Hq * kHeadDim;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-    // The tile is needed only if some unit's candidate range meets [b0, b0+64).
-    __shared__ int64_t s_lo[kLogitUnitRows], s_hi[kLogitUnitRows];
-    __shared__ int s_anchor[kLogitUnitRows];
-    __shared__ int any;
-    if (threadIdx.x == 0) any = 0;
+    // The tile is needed only if some unit's candidate range meets [b0, b0 + 128).
+    if (tid == 0) any = 0;
     __syncthreads();
-    if (threadIdx.x < units_per_tile) {
-        const int u = u0 + threadIdx.x;
-        int64_t lo = 0, hi = 0;
-        int anc = 0;
-        if (u < u_end) {
-            int64_t s, e;
-            unit_range(a.ut, u, &anc, &s, &e);
-            cand_range(a, s, &lo, &hi);
-        }
-        s_lo[threadIdx.x] = lo;
-        s_hi[threadIdx.x] = hi;
-        s_anchor[threadIdx.x] = anc;
-        if (lo < hi && lo < b0 + kLogitBlocks && hi > b0) atomicOr(&any, 1);
+    if (tid < n_u) {
+        int64_t s, e, lo, hi;
+        int anc;
+        unit_range(a.ut, u0 + tid, &anc, &s, &e);
+        cand_range(a, s, &lo, &hi);
+        s_lo[tid] = lo;
+        s_hi[tid] = hi;
+        s_anchor[tid] = anc;
+        if (lo < hi && lo < b0 + 128 && hi > b0) atomicOr(&any, 1);
     }
     __syncthreads();
     if (!any) return;
 
-    for (int i = threadIdx.x; i < rows * kHeadDim; i += blockDim.x) {
-        const int r = i / kHeadDim, d = i % kHeadDim;
-        const int ul = r / a.g;
-        const int h = j * a.g + r % a.g;
-        As[i] = (u0 + ul < u_end) ? fp[static_cast<int64_t>(s_anchor[ul]) * D + h * kHeadDim + d] : 0.f;
+    uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+    uint8_t* abuf = smem;                // A parts 0..2
+    uint8_t* bbuf = smem + 3 * kLtPart;  // B parts 0..2
+    // 128 rows x 32 float4 per operand; a warp reads one 512-byte row
+    for (int x = tid; x < 128 * 32; x += kLtThreads) {
+        const int r = x >> 5, c = (x & 31) * 4;
+        float4 va = make_float4(0.f, 0.f, 0.f, 0.f), vb = va;
+        if (r < rows) {
+            const int ul = r / a.g, hl = r % a.g;
+            va = *reinterpret_cast<const float4*>(fp + static_cast<int64_t>(s_anchor[ul]) * D +
+                                                  (j * a.g + hl) * kHeadDim + c);
+        }
+        if (b0 + r < a.nb) vb = *reinterpret_cast<const float4*>(reps + (j * a.nb + b0 + r) * kHeadDim + c);
+        put_split4(abuf, r, c, va);
+        put_split4(bbuf, r, c, vb);
     }
-    for (int i = threadIdx.x; i < kLogitBlocks * kHeadDim; i += blockDim.x) {
-        const int bb = i / kHeadDim, d = i % kHeadDim;
-        const int64_t b = b0 + bb;
-        Bs[bb * (kHeadDim + 1) + d] = (b < a.nb) ? reps[(static_cast<int64_t>(j) * a.nb + b) * kHeadDim + d] : 0.f;
+    fence_proxy_async_smem();
+    if (tid == 0) {
+        mbar_init(&d_full, 1);
+        fence_barrier_init();
     }
+    if (warp == 1) {
+        tmem_alloc(&tmem_slot, 128);
+        tmem_relinquish();
+    }
+    tc_fence_before();
     __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
 
-    const int tx = threadIdx.x % kLogitBlocks;
-    const int ty = threadIdx.x / kLogitBlocks;
-    const int64_t b = b0 + tx;
-    const float* bp = Bs + tx * (kHeadDim + 1);
-    for (int r = ty; r < rows; r += kLogitThreads / kLogitBlocks) {
-        const int ul = r / a.g;
-        if (u0 + ul >= u_end || b < s_lo[ul] || b >= s_hi[ul]) continue;
-        const float* ap = As + r * kHeadDim;
-        float acc = 0.f;
-#pragma unroll 8
-        for (int d = 0; d < kHeadDim; ++d) acc = fmaf(ap[d], bp[d], acc);
-        const int h = j * a.g + r % a.g;
-        logits[(static_cast<int64_t>(u0 + ul) * a.Hq + h) * a.nb + b] = a.sigma * acc;
+    if (tid == 0) {
+        const uint32_t idesc = idesc_bf16_f32(128, 128, 0);
+        const uint64_t ad = sdesc_sw128(smem_addr(abuf), 16, 1024);
+        const uint64_t bd = sdesc_sw128(smem_addr(bbuf), 16, 1024);
+        constexpr uint64_t kPartStep = kLtPart >> 4;
+        // (A part, B part): the products a_i b_j with i + j <= 4 (parts from 1)
+        constexpr int kPa[6] = {0, 0, 1, 0, 1, 2};
+        constexpr int kPb[6] = {0, 1, 0, 2, 1, 0};
+#pragma unroll
+        for (int i = 0; i < 6; ++i)
+            mma_ss_k128<kLtHalf>(tmem, ad + kPa[i] * kPartStep, bd + kPb[i] * kPartStep, idesc, i > 0 ? 1u : 0u);
+        mma_commit(&d_full);
+    }
+    bool done = true;
+    if (warp < 4) {
+        // epilogue: thread = row (TMEM lane) warp * 32 + lane
+        done = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&d_full, 0, a.timeout_ns, nullptr));
+        if (done) {
+            tc_fence_after();
+            const uint32_t lane_base = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+            uint32_t zr[128];
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc)
+                tmem_ld32(lane_base + cc * 32, *reinterpret_cast<uint32_t(*)[32]>(&zr[cc * 32]));
+            tmem_ld_wait();
+            const int r = warp * 32 + lane;
+            if (r < rows) {
+                const int ul = r / a.g, hl = r % a.g;
+                const int64_t lo = s_lo[ul] > b0 ? s_lo[ul] : b0;
+                const int64_t hi = s_hi[ul] < b0 + 128 ? s_hi[ul] : b0 + 128;
+                float* dst = logits + (static_cast<int64_t>(u0 + ul) * a.Hq + j * a.g + hl) * a.nb + b0;
+                const int c_lo = static_cast<int>(lo - b0), c_hi = static_cast<int>(hi - b0);
+#pragma unroll
+                for (int c = 0; c < 128; ++c)
+                    if (c >= c_lo && c < c_hi) dst[c] = a.sigma * __uint_as_float(zr[c]);
+            }
+        } else if (lane == 0) {
+            record_status(a.status, SCALE_ERR_TIMEOUT);
+        }
+    } else if (warp == 4 && lane == 0) {
+        // TMEM is freed only after the MMAs completed (bounded)
+        mbar_wait_bounded(&d_full, 0, a.timeout_ns, nullptr);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 128);
     }
 }
 
@@ -706,7 +806,7 @@ int topk_max_chunks(const Derived& d) { return static_cast<int>((d.nb + kChunk -
 cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t tok_end,
                           const float* reps, const float* fingerprints, const int32_t* unit_start,
                           const int32_t* n_units, int32_t* sel_blocks, int32_t* sel_count,
-                          float* sel_scores, uint8_t* ws, cudaStream_t st)
+                          float* sel_scores, uint8_t* ws, uint64_t timeout_ns, cudaStream_t st)
 {
     const WsLayout lay = ws_layout(d);
     float* logits = reinterpret_cast<float*>(ws + lay.logits);
@@ -725,17 +825,18 @@ cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t
     a.n_sink = d.n_sink;
     a.n_local = d.n_local;
     a.sigma = d.sigma;
+    a.status = reinterpret_cast<int32_t*>(ws + kStatusOffset);
+    a.timeout_ns = timeout_ns;
     const int max_units = a.sc_end - a.sc_begin;  // units in range <= sub-chunks in range
     if (max_units <= 0) return cudaSuccess;
 
-    const int upt = kLogitUnitRows / d.g;
-    const size_t smem = (kLogitUnitRows * kHeadDim + kLogitBlocks * (kHeadDim + 1)) * sizeof(float);
+    const int upt = 128 / d.g;  // units per logits tile
     // set on every launch: the attribute belongs to the current device
     cudaError_t e = cudaFuncSetAttribute(k_logits, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+                                         static_cast<int>(kLtSmem));
     if (e != cudaSuccess) return e;
-    dim3 gl((max_units + upt - 1) / upt, static_cast<unsigned>((d.nb + kLogitBlocks - 1) / kLogitBlocks), d.Hkv);
-    k_logits<<<gl, kLogitThreads, smem, st>>>(a, fingerprints, reps, logits);
+    dim3 gl((max_units + upt - 1) / upt, static_cast<unsigned>((d.nb + 127) / 128), d.Hkv);
+    k_logits<<<gl, kLtThreads, kLtSmem, st>>>(a, fingerprints, reps, logits);
     const int64_t rows = static_cast<int64_t>(max_units) * d.Hq;
     k_stats<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a, logits, stats);
     k_vote<<<dim3(static_cast<unsigned>((d.nb + 255) / 256), max_units), 256, 0, st>>>(a, logits, stats, scores);
