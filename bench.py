@@ -56,6 +56,9 @@ def parse_args():
                     help="keep K and V in a paged cache of P-token pages (shuffled page order)")
     ap.add_argument("--decode", action="store_true",
                     help="decode steps with the selection cache at the end of the context (one JSON line)")
+    ap.add_argument("--stage", choices=["select"], default=None,
+                    help="time one stage alone over the whole layer (one JSON line): 'select' = scale_select "
+                         "(steps (b)-(c)) after one step (a)")
     ap.add_argument("--sweep", action="store_true",
                     help="clustering-threshold sweep (theta x L_max) on planted-topic data: cluster sizes, "
                          "overlap ratio rho, boundary recall and step time (one JSON line)")
@@ -276,6 +279,14 @@ def selection_agreement(w, ref, sel, cnt) -> dict:
 # --------------------------------------------------------------------------- arms
 
 
+def workload_config(w, mode_name: str) -> dict:
+    """The workload keys of the JSON line's config, shared by both arms."""
+    return {"workload": w.name, "n_tokens": w.n_tokens, "q_heads": w.num_q_heads, "kv_heads": w.num_kv_heads,
+            "head_dim": w.head_dim, "sub_chunk": w.sub_chunk, "outer_chunk": w.outer_chunk,
+            "max_cluster_subchunks": w.max_cluster_subchunks, "block_size": w.block_size, "top_k": w.top_k,
+            "n_sink": w.n_sink, "n_local": w.n_local, "theta": w.theta, "mode": mode_name}
+
+
 def dist_setup(args):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -309,7 +320,7 @@ def run_reference(args):
         "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_run * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": w.name, "n_tokens": w.n_tokens, "mode": args.mode, "theta": w.theta},
+        "config": dict(workload_config(w, args.mode), parallelism="host cores (oracle)"),
         "extrapolated": last["extrapolated"], "rows_timed": last["rows"], "rows_total": w.n_tokens,
         "ms_per_step_extrapolated": t_full * 1e3,
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": last["cores"], "kind": "oracle",
@@ -507,11 +518,7 @@ def run_scale(args):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": w.name, "n_tokens": w.n_tokens, "q_heads": w.num_q_heads,
-                   "kv_heads": w.num_kv_heads, "head_dim": w.head_dim, "sub_chunk": w.sub_chunk,
-                   "outer_chunk": w.outer_chunk, "max_cluster_subchunks": w.max_cluster_subchunks,
-                   "block_size": w.block_size, "top_k": w.top_k, "n_sink": w.n_sink, "n_local": w.n_local,
-                   "theta": w.theta, "mode": mode_name, "parallelism": f"independent layers x{world}",
+        "config": {**workload_config(w, mode_name), "parallelism": f"independent layers x{world}",
                    "loop": ("Algorithm 2: per outer chunk scale_build_reps_range, then one scale_select and "
                             "one scale_sparse_prefill per unit (" +
                             ("sub-chunk" if per_sub else "cluster; one per outer chunk at theta = -1") + ")"),
@@ -950,10 +957,56 @@ def run_stack(args):
     return 0
 
 
+def run_stage(args):
+    """One stage of the path timed alone over the whole layer: scale_select
+    (steps (b) and (c): scoring of every unit's candidates, soft vote, top-k)
+    on the representatives and fingerprints of one step (a), in the chosen
+    mode; CUDA events around each call on the launch stream."""
+    import torch
+
+    import paper_2609_31568_gb300 as pkg
+    from paper_2609_31568_gb300 import scale as S
+
+    pkg.build()
+    S.load()
+    w = workload(args.workload)
+    mode = S.SCALE_MODE_PER_SUBCHUNK if args.mode == "subchunk" else S.SCALE_MODE_PER_CLUSTER
+    q, k, v = generate_layer(w)
+    dev = [torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k)]
+    del q, k, v
+    p = S.params_for(w)
+    buf = pkg.allocate(p, mode)
+    stream = torch.cuda.current_stream()
+    S.scale_build_reps(p, dev[0], dev[1], buf.reps, buf.fingerprints, buf.unit_start, buf.n_units, buf.ws, stream)
+    for _ in range(args.warmup):
+        S.select(p, mode, 0, w.n_tokens, dev[1], buf, stream)
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(args.steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        S.select(p, mode, 0, w.n_tokens, dev[1], buf, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    st = S.scale_get_device_status(buf.ws)
+    if st != S.SCALE_OK:
+        raise RuntimeError(f"device status {st}: {S.status_string(st)}")
+    n = w.n_subchunks if mode == S.SCALE_MODE_PER_SUBCHUNK else int(buf.n_units.item())
+    line = {"metric": "selection (steps (b)-(c)) time per call", "stage": "select", "unit": "us",
+            "value": statistics.median(times) * 1e3, "min": min(times) * 1e3, "steps": args.steps,
+            "warmup": args.warmup, "units": n, "config": workload_config(w, args.mode), "data": "synthetic",
+            "higher_is_better": False}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.stage:
+        return run_stage(args)
     if args.sweep:
         return run_sweep(args)
     if args.decode:
