@@ -950,6 +950,16 @@ def run_stack(args):
         per_sub_first = mode == S.SCALE_MODE_PER_SUBCHUNK
         line["scr_over_subchunk"] = (ms2 / ms) if per_sub_first else (ms / ms2)
         line["attn_flops_ratio"] = (flops2 / flops) if per_sub_first else (flops / flops2)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        # the oracle on layer 0 (steps (a)-(c) in full, Eq. 10 on the fixed row
+        # sample), extrapolated to every row of every layer
+        q0, k0, v0 = generate_layer(w, layer=0, seed=w.seed + 0)
+        r = oracle_sample(w, q0, k0, v0, mode == S.SCALE_MODE_PER_SUBCHUNK)
+        line["cpu_baseline"] = {
+            "value": r["tokens_per_s"] / w.layers, "unit": "tokens/s", "cores": r["cores"], "kind": "oracle",
+            "sample": f"layer 0 of {w.layers}: " + sample_label(w, r) + f"; times {w.layers} layers",
+            "extrapolated": True, "rows_timed": r["rows"], "rows_total": w.n_tokens * w.layers,
+            "ms_run": r["t_run"] * 1e3}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:

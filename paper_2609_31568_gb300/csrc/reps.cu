@@ -33,36 +33,51 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p)
 }
 
 // Representative key of block b for every KV head: the mean of the block's
-// keys. One CTA per block; thread c owns elements [8c, 8c+8) of the token row
-// (H_kv * 128 elements), so every token row is read as one coalesced span.
-// Grid: the blocks [b_base, b_base + gridDim.x).
+// keys. One CTA per block, `groups` row groups of row_chunks threads: thread
+// c of group g owns elements [8c, 8c+8) of the token rows g, g + groups, ...
+// of the block (every row read as one coalesced span), with 8 loads in
+// flight; the groups' sums are then added in group order, so the result is
+// bit-reproducible. Grid: the blocks [b_base, b_base + gridDim.x).
+constexpr int kRepGroups = 4;  // row groups when H_kv * 16 * 4 threads fit a CTA
+
 __global__ void __launch_bounds__(1024) k_block_reps(const uint4* __restrict__ k, KvPaging pg, int64_t N,
-                                                      int row_chunks, int B, int64_t nb, int64_t b_base,
-                                                      float* __restrict__ reps)
+                                                      int row_chunks, int groups, int B, int64_t nb,
+                                                      int64_t b_base, float* __restrict__ reps)
 {
-    const int c = threadIdx.x;
-    if (c >= row_chunks) return;
+    extern __shared__ float4 part[];  // [groups][row_chunks][2]
+    const int c = threadIdx.x % row_chunks;
+    const int g = threadIdx.x / row_chunks;
     const int64_t b = b_base + blockIdx.x;
     const int64_t t0 = b * B;
     const int64_t t1 = (t0 + B < N) ? t0 + B : N;
     float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
     const uint4* src = k + c;
     const uint4 zero = make_uint4(0, 0, 0, 0);
-    int64_t t = t0;
-    for (; t + 8 <= t1; t += 8) {
+    int64_t t = t0 + g;
+    for (; t + 7 * groups < t1; t += 8 * groups) {
         uint4 x[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-            const int64_t r = kv_row(pg, t + i);  // -1: a page outside the pool reads as zeros
+            const int64_t r = kv_row(pg, t + i * groups);  // -1: a page outside the pool reads as zeros
             x[i] = r < 0 ? zero : ld_stream(src + r * row_chunks);
         }
 #pragma unroll
         for (int i = 0; i < 8; ++i) add_bf16x8(acc, x[i]);
     }
-    for (; t < t1; ++t) {
+    for (; t < t1; t += groups) {
         const int64_t r = kv_row(pg, t);
         add_bf16x8(acc, r < 0 ? zero : ld_stream(src + r * row_chunks));
     }
+    part[(g * row_chunks + c) * 2] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+    part[(g * row_chunks + c) * 2 + 1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+    __syncthreads();
+    if (g != 0) return;
+    for (int gg = 1; gg < groups; ++gg) {
+        const float4 lo = part[(gg * row_chunks + c) * 2], hi = part[(gg * row_chunks + c) * 2 + 1];
+        acc[0] += lo.x; acc[1] += lo.y; acc[2] += lo.z; acc[3] += lo.w;
+        acc[4] += hi.x; acc[5] += hi.y; acc[6] += hi.z; acc[7] += hi.w;
+    }
+    // acc held group 0's sum; the groups are added in order for every element
     const float cnt = static_cast<float>(t1 - t0);
     const int j = c / (kHeadDim / 8);
     const int d0 = (c % (kHeadDim / 8)) * 8;
@@ -160,10 +175,19 @@ __global__ void k_gram(const float* __restrict__ fp, const float* __restrict__ s
     for (int d = warp + 1; d < S_max; d += nw) {
         const int j = i + d;
         if (j >= chunk_end) continue;
-        const float* a = fp + static_cast<int64_t>(i) * D;
-        const float* b = fp + static_cast<int64_t>(j) * D;
-        float s = 0.f;
-        for (int c = lane; c < D; c += 32) s = fmaf(a[c], b[c], s);
+        const float4* a = reinterpret_cast<const float4*>(fp + static_cast<int64_t>(i) * D);
+        const float4* b = reinterpret_cast<const float4*>(fp + static_cast<int64_t>(j) * D);
+        // 16-byte loads, four independent FMA chains (D is a multiple of 128)
+        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll 8
+        for (int c = lane; c < D / 4; c += 32) {
+            const float4 x = a[c], y = b[c];
+            s0 = fmaf(x.x, y.x, s0);
+            s1 = fmaf(x.y, y.y, s1);
+            s2 = fmaf(x.z, y.z, s2);
+            s3 = fmaf(x.w, y.w, s3);
+        }
+        float s = (s0 + s1) + (s2 + s3);
         for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
         const float na = fp_norm(ss_part, groups, i), nb = fp_norm(ss_part, groups, j);  // whole warp
         if (lane == 0) gram[static_cast<int64_t>(i) * S_max + d] = (na > 0.f && nb > 0.f) ? s / (na * nb) : 0.f;
@@ -275,9 +299,11 @@ cudaError_t launch_build_reps_range(const Derived& d, const void* q, const void*
     const int64_t b1 = t1 == d.N ? d.nb : t1 / d.B;
 
     const int row_chunks = d.Hkv * (kHeadDim / 8);
+    const int groups = row_chunks * kRepGroups <= 1024 ? kRepGroups : 1024 / row_chunks;
     if (reps && b1 > b0)  // block size 1 may skip them: token-level selection reads K itself
-        k_block_reps<<<static_cast<unsigned>(b1 - b0), row_chunks, 0, st>>>(
-            static_cast<const uint4*>(k), pg, d.N, row_chunks, d.B, d.nb, b0, reps);
+        k_block_reps<<<static_cast<unsigned>(b1 - b0), row_chunks * groups,
+                       static_cast<size_t>(groups) * row_chunks * 2 * sizeof(float4), st>>>(
+            static_cast<const uint4*>(k), pg, d.N, row_chunks, groups, d.B, d.nb, b0, reps);
 
     const int D8 = d.D / 8;
     const unsigned nm = static_cast<unsigned>(m1 - m0);
