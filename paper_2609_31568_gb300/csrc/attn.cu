@@ -80,7 +80,8 @@ struct AttnArgs {
 
 struct Barriers {
     uint64_t q_full;
-    uint64_t k_full[2], v_full[2], k_empty[2], v_empty[2];
+    uint64_t k_full[2], v_full[2];
+    uint64_t iter_done[2];  // [t & 1]: end of MMA iteration t: K(t) and V(t - 1) are free
     uint64_t s_full[2];  // S of Q tile q ready (and every earlier MMA of the CTA done)
     uint64_t p_full[2];  // P of Q tile q written (128 arrivals)
     uint64_t o_full;     // last P.V of both tiles done
@@ -149,8 +150,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars.k_full[i], 1);
             mbar_init(&bars.v_full[i], 1);
-            mbar_init(&bars.k_empty[i], 1);
-            mbar_init(&bars.v_empty[i], 1);
+            mbar_init(&bars.iter_done[i], 1);
             mbar_init(&bars.s_full[i], 1);
             mbar_init(&bars.p_full[i], 128);
         }
@@ -261,7 +261,8 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 // 64-row boxes: every one lies inside one KV page
                 const int32_t ra = packed ? 0 : kv_row_tma(a.pg, ta);
                 const int32_t rb = packed ? 0 : kv_row_tma(a.pg, tb);
-                if (t >= 2 && !mbar_wait_bounded(&bars.k_empty[st], ph, a.timeout_ns, &abort_flag)) {
+                // K(t) reuses the stage of K(t - 2): free at the end of iteration t - 2
+                if (t >= 2 && !mbar_wait_bounded(&bars.iter_done[st], ph, a.timeout_ns, &abort_flag)) {
                     fail(&abort_flag, a.status);
                     break;
                 }
@@ -276,7 +277,9 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                         tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.k_full[st], hf * 64, kvh, rb);
                     }
                 }
-                if (t >= 2 && !mbar_wait_bounded(&bars.v_empty[st], ph, a.timeout_ns, &abort_flag)) {
+                // V(t) reuses the stage of V(t - 2): free at the end of iteration t - 1
+                if (t >= 2 && !mbar_wait_bounded(&bars.iter_done[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns,
+                                                  &abort_flag)) {
                     fail(&abort_flag, a.status);
                     break;
                 }
@@ -322,12 +325,14 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
             };
             for (int t = 0; ok && t < T; ++t) {
                 const int st = t & 1;
-                if (!mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                if (!mbar_test(&bars.k_full[st], (t >> 1) & 1) &&
+                    !mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 for (int qt = 0; qt < 2; ++qt) {
                     if (t > 0) {
                         if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                        if (qt == 0 && !mbar_wait_bounded(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                        if (qt == 0 && !mbar_test(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1) &&
+                            !mbar_wait_bounded(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                         tc_fence_after();
                         issue_pv(t - 1, qt);
                     }
@@ -335,8 +340,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                     mma_commit(&bars.s_full[qt]);
                 }
                 if (!ok) break;
-                mma_commit(&bars.k_empty[st]);
-                if (t > 0) mma_commit(&bars.v_empty[(t - 1) & 1]);
+                mma_commit(&bars.iter_done[st]);  // K(t) and V(t - 1) read
             }
             if (ok) {
                 for (int qt = 0; qt < 2 && ok; ++qt) {
