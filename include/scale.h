@@ -50,8 +50,9 @@
  *    is no CPU fallback: every step runs in this library's CUDA kernels.
  *  - Concurrency. Calls are reentrant; two calls that share a workspace must
  *    not overlap on the GPU.
- *  - Supported shapes: head_dim 128, H_q / H_kv even (for the attention call),
- *    N < 2^31, outer_chunk a multiple of sub_chunk.
+ *  - Supported shapes: head_dim 128, H_q / H_kv at most 32 (at most 8 for
+ *    token-level selection and decode), H_kv at most 64, N < 2^31,
+ *    outer_chunk a multiple of sub_chunk.
  */
 #ifndef SCALE_H
 #define SCALE_H
@@ -200,8 +201,8 @@ int scale_select(const scale_params_t *p, int32_t mode, int64_t tok_begin, int64
  *   sel_tokens  int32 [M][top_k] out (ascending token indices, -1 padded)
  *   sel_count   int32 [M] out
  *   sel_scores  fp32 [M][N] or NULL: score_t on the candidates, NaN elsewhere.
- * Same range rule, modes and workspace as scale_select. H_q / H_kv must be 1,
- * 2, 4 or 8 (SCALE_ERR_UNSUPPORTED otherwise); block_size != 1 gives
+ * Same range rule, modes and workspace as scale_select. H_q / H_kv must be at
+ * most 8 (SCALE_ERR_UNSUPPORTED otherwise); block_size != 1 gives
  * SCALE_ERR_INVALID_ARG (and scale_select gives SCALE_ERR_UNSUPPORTED for
  * block size 1). */
 int scale_select_tokens(const scale_params_t *p, int32_t mode, int64_t tok_begin, int64_t tok_end,

@@ -335,7 +335,7 @@ static int select_tokens_impl(const Derived& d, int32_t mode, int64_t tok_begin,
 {
     int rc;
     if (d.B != 1) return SCALE_ERR_INVALID_ARG;
-    if (d.g != 1 && d.g != 2 && d.g != 4 && d.g != 8) return SCALE_ERR_UNSUPPORTED;
+    if (d.g > 8) return SCALE_ERR_UNSUPPORTED;  // token-level scoring: up to 8 query heads per KV head
     if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
     if (!device_ptr(k, 16) || !device_ptr(fingerprints, 16) || !device_ptr(sel_count, 4) ||
         (d.k > 0 && !device_ptr(sel_tokens, 4)) || (sel_scores && !device_ptr(sel_scores, 4)))
@@ -385,7 +385,6 @@ static int sparse_prefill_impl(const Derived& d, int32_t mode, int64_t tok_begin
 {
     int rc;
     if ((rc = check_range(d, mode, tok_begin, tok_end))) return rc;
-    if (d.g % 2) return SCALE_ERR_UNSUPPORTED;
     if (d.B > 1 && max_distant_segments(d) > kMaxSegments) return SCALE_ERR_UNSUPPORTED;
     if (!device_ptr(q, 16) || !device_ptr(k, 16) || !device_ptr(v, 16) || !device_ptr(out, 16) ||
         !device_ptr(sel_count, 4) || (d.k > 0 && !device_ptr(sel_blocks, 4)))

@@ -10,7 +10,9 @@
 // range and each selected block clipped to [n_sink, W_u), so every key is
 // visited once (the de-duplication of Sec. V-A3).
 //
-// Design (one CTA per work item = 128 query rows x 2 query heads of one KV head):
+// Design (one CTA per work item = 128 query rows x 2 query heads of one KV head;
+// with an odd number of query heads per KV head the last one of each group
+// runs alone, as a CTA with one query tile):
 //  - D_u is cut into 64-row segments; two segments form a 128-key tile. Each
 //    segment is one TMA box per 64-column half of head_dim, so gathered blocks
 //    land in shared memory in the 128-byte-swizzled K-major layout the tensor
@@ -121,6 +123,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     lin /= a.Hkv * a.pairs;
     const int kvh = hp / a.pairs;
     const int h0 = kvh * a.g + 2 * (hp % a.pairs);
+    const int nq = (h0 + 1 < (kvh + 1) * a.g) ? 2 : 1;  // query tiles (heads) of this CTA
     const int per_chunk = a.sc_per_chunk * a.qb_per_sc;
     const int c = lin / per_chunk;
     const int sc0 = a.sc_begin + c * a.sc_per_chunk;
@@ -236,8 +239,8 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 tma_prefetch_desc(&tpk);
                 tma_prefetch_desc(&tpv);
             }
-            mbar_arrive_expect_tx(&bars.q_full, 2 * kTileBytes);
-            for (int qt = 0; qt < 2; ++qt)
+            mbar_arrive_expect_tx(&bars.q_full, nq * kTileBytes);
+            for (int qt = 0; qt < nq; ++qt)
                 for (int hf = 0; hf < 2; ++hf)
                     tma_load_3d(smem + kOffQ + qt * kTileBytes + hf * kHalf, &tq, &bars.q_full,
                                 hf * 64, h0 + qt, static_cast<int32_t>(q0));
@@ -328,7 +331,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 if (!mbar_test(&bars.k_full[st], (t >> 1) & 1) &&
                     !mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                 tc_fence_after();
-                for (int qt = 0; qt < 2; ++qt) {
+                for (int qt = 0; qt < nq; ++qt) {
                     if (t > 0) {
                         if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                         if (qt == 0 && !mbar_test(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1) &&
@@ -343,7 +346,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 mma_commit(&bars.iter_done[st]);  // K(t) and V(t - 1) read
             }
             if (ok) {
-                for (int qt = 0; qt < 2 && ok; ++qt) {
+                for (int qt = 0; qt < nq && ok; ++qt) {
                     if (!mbar_wait_bounded(&bars.p_full[qt], (T - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                     if (qt == 0 && !mbar_wait_bounded(&bars.v_full[(T - 1) & 1], ((T - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                     tc_fence_after();
@@ -358,7 +361,7 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 mbar_wait_bounded(&bars.drain, 0, a.timeout_ns, nullptr);
             }
         }
-    } else {
+    } else if ((warp >> 2) < nq) {
         // ------------------------------------------------------------ softmax + epilogue
         const int qt = warp >> 2;
         const int quarter = warp & 3;
@@ -641,7 +644,7 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
     a.Hq = d.Hq;
     a.Hkv = d.Hkv;
     a.g = d.g;
-    a.pairs = d.g / 2;
+    a.pairs = (d.g + 1) / 2;  // an odd group's last head runs alone
     a.N = d.N;
     a.nb = d.nb;
     a.B = d.B;

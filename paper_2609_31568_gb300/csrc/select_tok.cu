@@ -470,7 +470,11 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
     switch (d.g) {
     case 1: e = run_tok_passes<1>(grid, rows, tf, tk, a, st); break;
     case 2: e = run_tok_passes<2>(grid, rows, tf, tk, a, st); break;
+    case 3: e = run_tok_passes<3>(grid, rows, tf, tk, a, st); break;
     case 4: e = run_tok_passes<4>(grid, rows, tf, tk, a, st); break;
+    case 5: e = run_tok_passes<5>(grid, rows, tf, tk, a, st); break;
+    case 6: e = run_tok_passes<6>(grid, rows, tf, tk, a, st); break;
+    case 7: e = run_tok_passes<7>(grid, rows, tf, tk, a, st); break;
     case 8: e = run_tok_passes<8>(grid, rows, tf, tk, a, st); break;
     default: return cudaErrorInvalidValue;
     }

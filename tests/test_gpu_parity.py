@@ -163,14 +163,16 @@ def _prefill_on(w, mode, dev, unit_start, n_units, sel, cnt, **over):
     ("gqa4-4k", dict(top_k=0, n_sink=0), 1),
     ("gqa4-4k", dict(block_size=256, top_k=2, n_sink=128, n_local=0), 1),
     ("llama8b-32k", GQA_SMALL, 5),
-    # query-head groups of 2 (one-CTA kernel) and 8 (CTA pairs, two head groups per KV head)
+    # query-head groups of 2, 8, 3 and 7 (the last head of an odd group runs
+    # in a CTA of its own with one query tile)
     ("gqa4-4k", dict(num_q_heads=8, num_kv_heads=4, n_tokens=2048 + 64), 1),
     ("gqa4-4k", dict(num_q_heads=16, num_kv_heads=2, n_tokens=2048 + 64), 1),
+    ("gqa4-4k", dict(num_q_heads=6, num_kv_heads=2, n_tokens=2048 + 64), 1),
+    ("gqa4-4k", dict(num_q_heads=7, num_kv_heads=1, n_tokens=2048 + 64), 1),
 ])
 def test_attention_parity_on_oracle_selection(name, over, stride, mode):
-    """scale_sparse_prefill on the oracle's selection vs the oracle's Eq. 10.
-    Query-head groups of a multiple of 4 run on CTA pairs, others on single
-    CTAs; both kernels are covered."""
+    """scale_sparse_prefill on the oracle's selection vs the oracle's Eq. 10,
+    for every row, including query-head groups of odd size."""
     w, q, k, v, dev = inputs(name, **over)
     rows = np.arange(0, w.n_tokens, stride)
     ref = oracle_path(w, q, k, v, mode, rows=rows)
@@ -179,6 +181,31 @@ def test_attention_parity_on_oracle_selection(name, over, stride, mode):
     got = to_f64_bf16(out[torch.from_numpy(rows).cuda()])
     mx, mean = attn_errors(got, ref["attn"])
     print(f"{name} {over} mode={mode}: max {mx:.3e} mean {mean:.3e}")
+    assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+def test_qwen2_7b_head_shape_end_to_end(mode):
+    """The head layout of the paper's model (Qwen2-7B: 28 query heads on 4 KV
+    heads, groups of 7) through all four steps: unit table, selection (exact
+    except near-ties) and every attention row against the oracle."""
+    w, q, k, v, dev = inputs("gqa4-4k", num_q_heads=28, num_kv_heads=4, n_tokens=2048 + 96)
+    p, buf = gpu_path(w, mode, dev)
+    ref = oracle_path(w, q, k, v, mode)
+    n = unit_count(buf, mode, w)
+    if mode == PER_CLUSTER:
+        assert buf.unit_start[: n + 1].cpu().numpy().tolist() == ref["unit_start"].tolist()
+    sel = buf.sel_blocks.cpu().numpy()[:n, : w.top_k]
+    same, near = compare_selection(sel, buf.sel_count.cpu().numpy()[:n], ref)
+    rows = np.arange(w.n_tokens)
+    us = ref["unit_start"] if mode == PER_CLUSTER else np.arange(w.n_subchunks + 1, dtype=np.int32)
+    ref_attn = oracle.attention_rows(q=q, k=k, v=v, sub_chunk=w.sub_chunk, block_size=w.block_size,
+                                     top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                                     attn_scale=1.0 / np.sqrt(w.head_dim), per_subchunk=(mode == PER_SUB),
+                                     unit_start=ref["unit_start"], sel=selection_for_reference(sel, ref, same),
+                                     sel_count=ref["sel_count"], rows=rows)
+    mx, mean = attn_errors(to_f64_bf16(buf.out), ref_attn)
+    print(f"28q/4kv mode={mode}: {n} units, {near} near-ties, max {mx:.3e} mean {mean:.3e} ({len(us) - 1} units)")
     assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
 
 
@@ -257,7 +284,10 @@ def test_end_to_end_parity_sampled(name, n_random, heavy, mode):
 
 TOKEN_CASES = [("gqa4-4k", dict(block_size=1, top_k=64)),
                ("gqa4-4k", dict(block_size=1, n_tokens=3000, n_sink=40, n_local=100, top_k=50)),
-               ("llama8b-32k", dict(block_size=1, top_k=1024))]
+               ("llama8b-32k", dict(block_size=1, top_k=1024)),
+               # the paper's model and selection: Qwen2-7B heads (28 on 4 KV heads), token level
+               ("gqa4-4k", dict(block_size=1, top_k=128, num_q_heads=28, num_kv_heads=4, n_tokens=2048 + 64)),
+               ("gqa4-4k", dict(block_size=1, top_k=96, num_q_heads=6, num_kv_heads=2, n_tokens=2048 + 64))]
 
 
 @pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
@@ -526,9 +556,9 @@ def test_invalid_arguments_are_rejected_before_launch():
         S.scale_sparse_prefill(p, PER_CLUSTER, 100, w.n_tokens, *dev, buf.unit_start, buf.n_units,
                                buf.sel_blocks, buf.sel_count, buf.out, buf.ws)
     assert e.value.rc == S.SCALE_ERR_INVALID_ARG
-    odd = S.params_for(w, num_q_heads=3, num_kv_heads=1)
+    narrow = S.params_for(w, head_dim=64)  # valid, but the kernels implement head_dim 128 only
     with pytest.raises(S.ScaleError) as e:
-        S.scale_sparse_prefill(odd, PER_SUB, 0, w.n_tokens, *dev, None, None, buf.sel_blocks,
+        S.scale_sparse_prefill(narrow, PER_SUB, 0, w.n_tokens, *dev, None, None, buf.sel_blocks,
                                buf.sel_count, buf.out, buf.ws)
     assert e.value.rc == S.SCALE_ERR_UNSUPPORTED
     torch.cuda.synchronize()
