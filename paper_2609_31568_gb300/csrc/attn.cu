@@ -96,6 +96,9 @@ __device__ __forceinline__ void fail(volatile int* abort_flag, int32_t* status)
     record_status(status, SCALE_ERR_TIMEOUT);
 }
 
+// Compile-time query-tile count (1 or 2) for the MMA issue loop.
+template <int N> struct TileCount { static constexpr int value = N; };
+
 // TOK: block size 1. The distant keys and values of each (unit, KV head)
 // were packed by k_tok_pack into contiguous rows [M * H_kv][slots][128]
 // (zero rows after the last one), so their tiles are plain TMA boxes of the
@@ -326,34 +329,41 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 mma_ts_k128<2048>(tmem + qt * 256 + 128, tmem + qt * 256, vdesc0 + (t & 1) * kStageStep, id_pv,
                                   t > 0 ? 1u : 0u);
             };
-            for (int t = 0; ok && t < T; ++t) {
-                const int st = t & 1;
-                if (!mbar_test(&bars.k_full[st], (t >> 1) & 1) &&
-                    !mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                tc_fence_after();
-                for (int qt = 0; qt < nq; ++qt) {
-                    if (t > 0) {
-                        if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                        if (qt == 0 && !mbar_test(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1) &&
-                            !mbar_wait_bounded(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                        tc_fence_after();
-                        issue_pv(t - 1, qt);
-                    }
-                    mma_ss_k128<kHalf>(tmem + qt * 256, qdesc0 + qt * kStageStep, kdesc0 + st * kStageStep, id_qk, 0u);
-                    mma_commit(&bars.s_full[qt]);
-                }
-                if (!ok) break;
-                mma_commit(&bars.iter_done[st]);  // K(t) and V(t - 1) read
-            }
-            if (ok) {
-                for (int qt = 0; qt < nq && ok; ++qt) {
-                    if (!mbar_wait_bounded(&bars.p_full[qt], (T - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                    if (qt == 0 && !mbar_wait_bounded(&bars.v_full[(T - 1) & 1], ((T - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+            // The query-tile count is a compile-time constant of the issue loop: this
+            // thread is the critical path, and a runtime bound costs ~10%.
+            auto issue_all = [&](auto nq_c) {
+                constexpr int NQ = decltype(nq_c)::value;
+                for (int t = 0; ok && t < T; ++t) {
+                    const int st = t & 1;
+                    if (!mbar_test(&bars.k_full[st], (t >> 1) & 1) &&
+                        !mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                     tc_fence_after();
-                    issue_pv(T - 1, qt);
+                    for (int qt = 0; qt < NQ; ++qt) {
+                        if (t > 0) {
+                            if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                            if (qt == 0 && !mbar_test(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1) &&
+                                !mbar_wait_bounded(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                            tc_fence_after();
+                            issue_pv(t - 1, qt);
+                        }
+                        mma_ss_k128<kHalf>(tmem + qt * 256, qdesc0 + qt * kStageStep, kdesc0 + st * kStageStep, id_qk, 0u);
+                        mma_commit(&bars.s_full[qt]);
+                    }
+                    if (!ok) break;
+                    mma_commit(&bars.iter_done[st]);  // K(t) and V(t - 1) read
                 }
-                if (ok) mma_commit(&bars.o_full);
-            }
+                if (ok) {
+                    for (int qt = 0; qt < NQ && ok; ++qt) {
+                        if (!mbar_wait_bounded(&bars.p_full[qt], (T - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                        if (qt == 0 && !mbar_wait_bounded(&bars.v_full[(T - 1) & 1], ((T - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                        tc_fence_after();
+                        issue_pv(T - 1, qt);
+                    }
+                    if (ok) mma_commit(&bars.o_full);
+                }
+            };
+            if (nq == 2) issue_all(TileCount<2>{});
+            else issue_all(TileCount<1>{});
             if (!ok) {
                 fail(&abort_flag, a.status);
                 // Drain: every MMA issued so far completes before TMEM is freed.
