@@ -18,13 +18,18 @@
 //    land in shared memory in the 128-byte-swizzled K-major layout the tensor
 //    cores read, with no copy through registers.
 //  - warp 8 (one thread) issues TMA loads: both Q tiles once, then K and V
-//    tiles into a 2-stage ring;
+//    tiles into a 2-stage ring, K(t) and V(t - 1) on one barrier;
 //  - warp 9 (one thread) issues tcgen05.mma: S_q = Q_q K^T into TMEM, and
-//    O_q += P_q V with P read from TMEM (bf16, written over S_q);
+//    O_q += P_q V with P read from TMEM (bf16, written over S_q). This thread
+//    bounds the kernel: every barrier operation it runs between two MMA
+//    groups leaves the tensor pipe idle, so it runs as few as it can (one
+//    K/V wait, and per query tile one P wait, one fence and one commit per
+//    key tile; the producer reuses the S-ready commits to free its stages);
 //  - warps 0-3 and 4-7 run the online softmax of Q tile 0 and 1, one thread
 //    per row (= TMEM lane), and the epilogue. The running max is raised only
 //    when it grows by more than 8 (log2 units), so O is rescaled rarely; the
 //    final normalisation uses the same max, which keeps the result exact.
+//    Most tiles skip the row max altogether (see the fast path below).
 //  - Every wait is bounded in wall time; on expiry the kernel records
 //    SCALE_ERR_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and
 //    returns.
@@ -45,6 +50,7 @@ constexpr uint32_t kTileBytes = 128 * 128 * 2;  // one 128 x 128 bf16 tile
 constexpr uint32_t kHalf = kTileBytes / 2;    // one 64-column half (128 rows x 128 B)
 constexpr uint32_t kSegBytes = 64 * 128;      // one 64-row x 64-column box
 constexpr float kRescaleThreshold = 8.0f;     // log2 units
+constexpr float kFastSumLimit = 65536.0f;     // 2^16: largest tile sum kept on the fast path
 // Softmax exponentials of column pair i go to the FMA pipe (exp2_poly2) when
 // bit (i % 8) is set, else to the special-function unit; the split balances
 // the two units, which otherwise bound the softmax.
@@ -82,9 +88,8 @@ struct AttnArgs {
 
 struct Barriers {
     uint64_t q_full;
-    uint64_t k_full[2], v_full[2];
-    uint64_t iter_done[2];  // [t & 1]: end of MMA iteration t: K(t) and V(t - 1) are free
-    uint64_t s_full[2];  // S of Q tile q ready (and every earlier MMA of the CTA done)
+    uint64_t kv_full[2];    // [t & 1]: K(t) and V(t - 1) landed (step T: V(T - 1) alone)
+    uint64_t s_full[2][2];  // [q][t & 1]: S(t) of Q tile q ready (and every earlier MMA of the CTA done)
     uint64_t p_full[2];  // P of Q tile q written (128 arrivals)
     uint64_t o_full;     // last P.V of both tiles done
     uint64_t drain;
@@ -154,10 +159,9 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
         abort_flag = 0;
         mbar_init(&bars.q_full, 1);
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&bars.k_full[i], 1);
-            mbar_init(&bars.v_full[i], 1);
-            mbar_init(&bars.iter_done[i], 1);
-            mbar_init(&bars.s_full[i], 1);
+            mbar_init(&bars.kv_full[i], 1);
+            mbar_init(&bars.s_full[i][0], 1);
+            mbar_init(&bars.s_full[i][1], 1);
             mbar_init(&bars.p_full[i], 128);
         }
         mbar_init(&bars.o_full, 1);
@@ -248,67 +252,72 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                     tma_load_3d(smem + kOffQ + qt * kTileBytes + hf * kHalf, &tq, &bars.q_full,
                                 hf * 64, h0 + qt, static_cast<int32_t>(q0));
             const int32_t prow = u * a.Hkv + kvh;  // packed (unit, KV head) plane
-            int issued_k0 = 0, issued_k1 = 0, issued_v0 = 0, issued_v1 = 0;
-            for (int t = 0; t < T && !abort_flag; ++t) {
+            // Step t (0..T) loads K(t) and V(t - 1) on kv_full[t & 1]; both stages
+            // they reuse were last read by MMAs of iteration t - 2 (Q K^T of K(t - 2),
+            // P.V of V(t - 3)), which the S-ready commit of the CTA's last query
+            // tile in that iteration covers.
+            uint64_t* const s_last = bars.s_full[nq - 1];
+            int issued0 = 0, issued1 = 0;
+            int32_t pa = 0, pb = 0;  // TMA rows of tile t - 1 (its V goes out at step t)
+            bool p_packed = false;
+            int32_t p_ta = 0;
+            for (int t = 0; t <= T && !abort_flag; ++t) {
                 const int st = t & 1;
-                const uint32_t ph = ((t >> 1) - 1) & 1;
-                const bool packed = TOK && t < n_dt;
-                int32_t ta, tb;
-                if (packed) {
-                    ta = 128 * t;
-                    tb = 0;
-                } else if (t < n_dt) {
-                    ta = seg[2 * t].x;
-                    tb = seg[2 * t + 1].x;
-                } else {
-                    ta = static_cast<int32_t>(W + 128ll * (t - n_dt));
-                    tb = ta + 64;
-                }
-                // 64-row boxes: every one lies inside one KV page
-                const int32_t ra = packed ? 0 : kv_row_tma(a.pg, ta);
-                const int32_t rb = packed ? 0 : kv_row_tma(a.pg, tb);
-                // K(t) reuses the stage of K(t - 2): free at the end of iteration t - 2
-                if (t >= 2 && !mbar_wait_bounded(&bars.iter_done[st], ph, a.timeout_ns, &abort_flag)) {
+                if (t >= 2 && !mbar_wait_bounded(&s_last[st], ((t - 2) >> 1) & 1, a.timeout_ns, &abort_flag)) {
                     fail(&abort_flag, a.status);
                     break;
                 }
-                mbar_arrive_expect_tx(&bars.k_full[st], kTileBytes);
-                if (st) ++issued_k1; else ++issued_k0;
-                uint8_t* kd = smem + kOffK + st * kTileBytes;
-                for (int hf = 0; hf < 2; ++hf) {
-                    if (packed) {
-                        tma_load_3d(kd + hf * kHalf, &tpk, &bars.k_full[st], hf * 64, ta, prow);
-                    } else {
-                        tma_load_3d(kd + hf * kHalf, &tk, &bars.k_full[st], hf * 64, kvh, ra);
-                        tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.k_full[st], hf * 64, kvh, rb);
+                const bool has_k = t < T, has_v = t >= 1;
+                mbar_arrive_expect_tx(&bars.kv_full[st], (has_k ? kTileBytes : 0u) + (has_v ? kTileBytes : 0u));
+                if (st) ++issued1; else ++issued0;
+                if (has_v) {
+                    uint8_t* vd = smem + kOffV + ((t - 1) & 1) * kTileBytes;
+                    for (int hf = 0; hf < 2; ++hf) {
+                        if (p_packed) {
+                            tma_load_3d(vd + hf * kHalf, &tpv, &bars.kv_full[st], hf * 64, p_ta, prow);
+                        } else {
+                            tma_load_3d(vd + hf * kHalf, &tv, &bars.kv_full[st], hf * 64, kvh, pa);
+                            tma_load_3d(vd + hf * kHalf + kSegBytes, &tv, &bars.kv_full[st], hf * 64, kvh, pb);
+                        }
                     }
                 }
-                // V(t) reuses the stage of V(t - 2): free at the end of iteration t - 1
-                if (t >= 2 && !mbar_wait_bounded(&bars.iter_done[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns,
-                                                  &abort_flag)) {
-                    fail(&abort_flag, a.status);
-                    break;
-                }
-                mbar_arrive_expect_tx(&bars.v_full[st], kTileBytes);
-                if (st) ++issued_v1; else ++issued_v0;
-                uint8_t* vd = smem + kOffV + st * kTileBytes;
-                for (int hf = 0; hf < 2; ++hf) {
+                if (has_k) {
+                    const bool packed = TOK && t < n_dt;
+                    int32_t ta, tb;
                     if (packed) {
-                        tma_load_3d(vd + hf * kHalf, &tpv, &bars.v_full[st], hf * 64, ta, prow);
+                        ta = 128 * t;
+                        tb = 0;
+                    } else if (t < n_dt) {
+                        ta = seg[2 * t].x;
+                        tb = seg[2 * t + 1].x;
                     } else {
-                        tma_load_3d(vd + hf * kHalf, &tv, &bars.v_full[st], hf * 64, kvh, ra);
-                        tma_load_3d(vd + hf * kHalf + kSegBytes, &tv, &bars.v_full[st], hf * 64, kvh, rb);
+                        ta = static_cast<int32_t>(W + 128ll * (t - n_dt));
+                        tb = ta + 64;
                     }
+                    // 64-row boxes: every one lies inside one KV page
+                    const int32_t ra = packed ? 0 : kv_row_tma(a.pg, ta);
+                    const int32_t rb = packed ? 0 : kv_row_tma(a.pg, tb);
+                    uint8_t* kd = smem + kOffK + st * kTileBytes;
+                    for (int hf = 0; hf < 2; ++hf) {
+                        if (packed) {
+                            tma_load_3d(kd + hf * kHalf, &tpk, &bars.kv_full[st], hf * 64, ta, prow);
+                        } else {
+                            tma_load_3d(kd + hf * kHalf, &tk, &bars.kv_full[st], hf * 64, kvh, ra);
+                            tma_load_3d(kd + hf * kHalf + kSegBytes, &tk, &bars.kv_full[st], hf * 64, kvh, rb);
+                        }
+                    }
+                    pa = ra;
+                    pb = rb;
+                    p_packed = packed;
+                    p_ta = ta;
                 }
             }
             if (abort_flag) {
                 // Drain: wait (bounded, ignoring the abort flag) for the last
                 // phase of every buffer that received copies.
                 mbar_wait_bounded(&bars.q_full, 0, a.timeout_ns, nullptr);
-                if (issued_k0) mbar_wait_bounded(&bars.k_full[0], (issued_k0 - 1) & 1, a.timeout_ns, nullptr);
-                if (issued_k1) mbar_wait_bounded(&bars.k_full[1], (issued_k1 - 1) & 1, a.timeout_ns, nullptr);
-                if (issued_v0) mbar_wait_bounded(&bars.v_full[0], (issued_v0 - 1) & 1, a.timeout_ns, nullptr);
-                if (issued_v1) mbar_wait_bounded(&bars.v_full[1], (issued_v1 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued0) mbar_wait_bounded(&bars.kv_full[0], (issued0 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued1) mbar_wait_bounded(&bars.kv_full[1], (issued1 - 1) & 1, a.timeout_ns, nullptr);
             }
         }
     } else if (warp == 9) {
@@ -335,27 +344,25 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                 constexpr int NQ = decltype(nq_c)::value;
                 for (int t = 0; ok && t < T; ++t) {
                     const int st = t & 1;
-                    if (!mbar_test(&bars.k_full[st], (t >> 1) & 1) &&
-                        !mbar_wait_bounded(&bars.k_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                    tc_fence_after();
+                    if (!mbar_test(&bars.kv_full[st], (t >> 1) & 1) &&
+                        !mbar_wait_bounded(&bars.kv_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                    // TMA data is ordered by the barrier's transaction count; from t = 1
+                    // the fence after the P wait below precedes every MMA of the iteration.
+                    if (t == 0) tc_fence_after();
                     for (int qt = 0; qt < NQ; ++qt) {
                         if (t > 0) {
                             if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                            if (qt == 0 && !mbar_test(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1) &&
-                                !mbar_wait_bounded(&bars.v_full[(t - 1) & 1], ((t - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                             tc_fence_after();
                             issue_pv(t - 1, qt);
                         }
                         mma_ss_k128<kHalf>(tmem + qt * 256, qdesc0 + qt * kStageStep, kdesc0 + st * kStageStep, id_qk, 0u);
-                        mma_commit(&bars.s_full[qt]);
+                        mma_commit(&bars.s_full[qt][st]);
                     }
-                    if (!ok) break;
-                    mma_commit(&bars.iter_done[st]);  // K(t) and V(t - 1) read
                 }
                 if (ok) {
+                    if (!mbar_wait_bounded(&bars.kv_full[T & 1], (T >> 1) & 1, a.timeout_ns, &abort_flag)) ok = false;
                     for (int qt = 0; qt < NQ && ok; ++qt) {
                         if (!mbar_wait_bounded(&bars.p_full[qt], (T - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                        if (qt == 0 && !mbar_wait_bounded(&bars.v_full[(T - 1) & 1], ((T - 1) >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                         tc_fence_after();
                         issue_pv(T - 1, qt);
                     }
@@ -382,13 +389,9 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
         const uint32_t o_addr = s_addr + 128;
         float m_run = -INFINITY, l_run = 0.f;
         bool ok = true;
-        for (int t = 0; t < T; ++t) {
-            // tcgen05.ld/st are warp-collective: the outcome must be warp-uniform.
-            const bool got = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.s_full[qt], t & 1, a.timeout_ns, &abort_flag));
-            if (!got) { ok = false; break; }
-            tc_fence_after();
-            // S row: four 32-column TMEM loads in flight, one wait.
-            uint32_t sr[128];
+        // S row of tile t: four 32-column TMEM loads in flight, one wait, then
+        // the keys outside the row's key set set to -inf.
+        auto load_s = [&](uint32_t (&sr)[128], int t) {
 #pragma unroll
             for (int c = 0; c < 4; ++c)
                 tmem_ld32(s_addr + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
@@ -417,63 +420,104 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
                         if (c > lim) s[c] = -INFINITY;
                 }
             }
-            // Row max: eight independent three-input max chains.
-            float mx8[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) mx8[i] = s[i];
-#pragma unroll
-            for (int c = 8; c < 120; c += 16)
-#pragma unroll
-                for (int i = 0; i < 8; ++i) mx8[i] = fmax3(mx8[i], s[c + 2 * i], s[c + 2 * i + 1]);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[120 + i]);
-            const float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
-                                   fmaxf(mx8[6], mx8[7]));
-            const float m_new = fmaxf(m_run, mx * a.scale_log2);
-            const bool raise = m_new > m_run + kRescaleThreshold;
-            // The O rescale goes through warp-collective TMEM loads and stores,
-            // so the branch is taken by the whole warp when any row needs it;
-            // rows that do not keep their max and scale by 1.
-            if (__any_sync(0xFFFFFFFFu, raise)) {
-                const float alpha = raise ? ex2(m_run - m_new) : 1.0f;
-                l_run *= alpha;
-                if (t > 0) {
-#pragma unroll 1
-                    for (int c = 0; c < 8; ++c) {
-                        uint32_t v[16];
-                        tmem_ld16(o_addr + c * 16, v);
-                        tmem_ld_wait();
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
-                        tmem_st16(o_addr + c * 16, v);
-                    }
-                }
-                if (raise) m_run = m_new;
-            }
-            const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
-            // p = 2^(s * scale_log2 - m): packed FMA, then the exponential.
+        };
+        // p = 2^(s * scale_log2 - m) for keys [64 h, 64 h + 64): packed FMA, then
+        // the exponential, packed to bf16 pairs in pk; returns the sum of the p.
+        auto exp_half = [&](const float* s, int h, float neg_m, uint32_t (&pk)[32]) {
             float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                uint32_t pk[32];
-#pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    float x0, x1;
-                    ffma2(x0, x1, s[h * 64 + 2 * i], s[h * 64 + 2 * i + 1], a.scale_log2, a.scale_log2,
-                          neg_m, neg_m);
-                    if ((kSoftExpMask >> (i & 7)) & 1u) {
-                        exp2_poly2(x0, x1, x0, x1);
-                    } else {
-                        x0 = ex2(x0);
-                        x1 = ex2(x1);
-                    }
-                    const int j = (i & 3) * 2;
-                    fadd2(acc[j], acc[j + 1], acc[j], acc[j + 1], x0, x1);
-                    pk[i] = pack_bf16x2(x0, x1);
+            for (int i = 0; i < 32; ++i) {
+                float x0, x1;
+                ffma2(x0, x1, s[h * 64 + 2 * i], s[h * 64 + 2 * i + 1], a.scale_log2, a.scale_log2, neg_m,
+                      neg_m);
+                if ((kSoftExpMask >> (i & 7)) & 1u) {
+                    exp2_poly2(x0, x1, x0, x1);
+                } else {
+                    x0 = ex2(x0);
+                    x1 = ex2(x1);
                 }
-                tmem_st32(s_addr + h * 32, pk);
+                const int j = (i & 3) * 2;
+                fadd2(acc[j], acc[j + 1], acc[j], acc[j + 1], x0, x1);
+                pk[i] = pack_bf16x2(x0, x1);
             }
-            const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+            return ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+        };
+        for (int t = 0; t < T; ++t) {
+            // tcgen05.ld/st are warp-collective: the outcome must be warp-uniform.
+            const bool got = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.s_full[qt][t & 1], (t >> 1) & 1, a.timeout_ns, &abort_flag));
+            if (!got) { ok = false; break; }
+            tc_fence_after();
+            float sum = 0.f;
+            // Fast path: the exponentials are taken against the running max as it
+            // stands, without the row max. The max only matters when the tile
+            // outgrows m_run by more than the raise threshold, and the sum shows
+            // it: a sum above 2^16 over 128 keys needs a term above 2^9, i.e. a
+            // logit more than 9 (log2 units) above m_run. Below that every p is
+            // at most 2^16, far inside the fp32 and bf16 ranges, so m_run may
+            // stay; a sum that is inf or NaN fails the test as well. The first
+            // tile (m_run = -inf) and every failed tile take the exact path on a
+            // fresh copy of S (nothing has been stored over it yet).
+            bool exact = !__all_sync(0xFFFFFFFFu, m_run != -INFINITY);
+            if (!exact) {
+                uint32_t sr[128];
+                load_s(sr, t);
+                const float* s = reinterpret_cast<const float*>(sr);
+                uint32_t pk[2][32];
+                const float sum0 = exp_half(s, 0, -m_run, pk[0]);
+                const float sum1 = exp_half(s, 1, -m_run, pk[1]);
+                sum = sum0 + sum1;
+                exact = __any_sync(0xFFFFFFFFu, !(sum <= kFastSumLimit));
+                if (!exact) {
+                    tmem_st32(s_addr, pk[0]);
+                    tmem_st32(s_addr + 32, pk[1]);
+                }
+            }
+            if (exact) {
+                sum = 0.f;
+                uint32_t sr[128];
+                load_s(sr, t);
+                const float* s = reinterpret_cast<const float*>(sr);
+                // Row max: eight independent three-input max chains.
+                float mx8[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+                for (int c = 8; c < 120; c += 16)
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) mx8[i] = fmax3(mx8[i], s[c + 2 * i], s[c + 2 * i + 1]);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[120 + i]);
+                const float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
+                                       fmaxf(mx8[6], mx8[7]));
+                const float m_new = fmaxf(m_run, mx * a.scale_log2);
+                const bool raise = m_new > m_run + kRescaleThreshold;
+                // The O rescale goes through warp-collective TMEM loads and stores,
+                // so the branch is taken by the whole warp when any row needs it;
+                // rows that do not keep their max and scale by 1.
+                if (__any_sync(0xFFFFFFFFu, raise)) {
+                    const float alpha = raise ? ex2(m_run - m_new) : 1.0f;
+                    l_run *= alpha;
+                    if (t > 0) {
+#pragma unroll 1
+                        for (int c = 0; c < 8; ++c) {
+                            uint32_t v[16];
+                            tmem_ld16(o_addr + c * 16, v);
+                            tmem_ld_wait();
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+                            tmem_st16(o_addr + c * 16, v);
+                        }
+                    }
+                    if (raise) m_run = m_new;
+                }
+                const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t pk[32];
+                    sum += exp_half(s, h, neg_m, pk);
+                    tmem_st32(s_addr + h * 32, pk);
+                }
+            }
             l_run += sum;
             tmem_st_wait();
             tc_fence_before();
