@@ -101,8 +101,66 @@ __device__ __forceinline__ void fail(volatile int* abort_flag, int32_t* status)
     record_status(status, SCALE_ERR_TIMEOUT);
 }
 
-// Compile-time query-tile count (1 or 2) for the MMA issue loop.
-template <int N> struct TileCount { static constexpr int value = N; };
+// One iteration t (t & 1 = ST) of the MMA issue loop of a CTA with NQ (1 or 2)
+// query tiles: wait for K(t) and V(t - 1), then per query tile wait for
+// P(t - 1), issue O += P(t - 1) V(t - 1) and S = Q K(t)^T, and commit S-ready.
+template <int NQ, int ST>
+__device__ __forceinline__ bool mma_iteration(Barriers* bars, uint32_t tmem, uint64_t qdesc0, uint64_t kdesc0,
+                                              uint64_t vdesc0, uint32_t id_qk, uint32_t id_pv, int t,
+                                              uint64_t timeout_ns, const volatile int* abort_flag)
+{
+    // Descriptors of the two stages differ by kTileBytes >> 4 in the address field.
+    constexpr uint64_t kStageStep = kTileBytes >> 4;
+    const uint32_t ph = (t >> 1) & 1;
+    if (!mbar_test(&bars->kv_full[ST], ph) && !mbar_wait_bounded(&bars->kv_full[ST], ph, timeout_ns, abort_flag))
+        return false;
+    // TMA data is ordered by the barrier's transaction count; from t = 1
+    // the fence after the P wait below precedes every MMA of the iteration.
+    if (t == 0) tc_fence_after();
+#pragma unroll
+    for (int qt = 0; qt < NQ; ++qt) {
+        if (t > 0) {
+            if (!mbar_wait_bounded(&bars->p_full[qt], ST ^ 1, timeout_ns, abort_flag)) return false;
+            tc_fence_after();
+            mma_ts_k128<2048>(tmem + qt * 256 + 128, tmem + qt * 256, vdesc0 + (ST ^ 1) * kStageStep, id_pv,
+                              t > 1 ? 1u : 0u);
+        }
+        mma_ss_k128<kHalf>(tmem + qt * 256, qdesc0 + qt * kStageStep, kdesc0 + ST * kStageStep, id_qk, 0u);
+        mma_commit(&bars->s_full[qt][ST]);
+    }
+    return true;
+}
+
+// The MMA issue loop, run by one thread: T iterations (two per trip, so the
+// stage indices are constants), then the last P.V and the O-ready commit.
+// This thread is the critical path: NQ is a compile-time constant and all
+// state is held in registers. Returns false when a wait ran out or the
+// kernel was aborted.
+template <int NQ>
+__device__ __forceinline__ bool mma_issue_loop(Barriers* bars, uint32_t tmem, uint64_t qdesc0, uint64_t kdesc0,
+                                               uint64_t vdesc0, uint32_t id_qk, uint32_t id_pv, int T,
+                                               uint64_t timeout_ns, const volatile int* abort_flag)
+{
+    constexpr uint64_t kStageStep = kTileBytes >> 4;
+    int t = 0;
+    for (; t + 1 < T; t += 2) {
+        if (!mma_iteration<NQ, 0>(bars, tmem, qdesc0, kdesc0, vdesc0, id_qk, id_pv, t, timeout_ns, abort_flag) ||
+            !mma_iteration<NQ, 1>(bars, tmem, qdesc0, kdesc0, vdesc0, id_qk, id_pv, t + 1, timeout_ns, abort_flag))
+            return false;
+    }
+    if (t < T && !mma_iteration<NQ, 0>(bars, tmem, qdesc0, kdesc0, vdesc0, id_qk, id_pv, t, timeout_ns, abort_flag))
+        return false;
+    if (!mbar_wait_bounded(&bars->kv_full[T & 1], (T >> 1) & 1, timeout_ns, abort_flag)) return false;
+#pragma unroll
+    for (int qt = 0; qt < NQ; ++qt) {
+        if (!mbar_wait_bounded(&bars->p_full[qt], (T - 1) & 1, timeout_ns, abort_flag)) return false;
+        tc_fence_after();
+        mma_ts_k128<2048>(tmem + qt * 256 + 128, tmem + qt * 256, vdesc0 + ((T - 1) & 1) * kStageStep, id_pv,
+                          T > 1 ? 1u : 0u);
+    }
+    mma_commit(&bars->o_full);
+    return true;
+}
 
 // TOK: block size 1. The distant keys and values of each (unit, KV head)
 // were packed by k_tok_pack into contiguous rows [M * H_kv][slots][128]
@@ -329,48 +387,14 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
             const uint32_t k_base = smem_addr(smem + kOffK);
             const uint32_t v_base = smem_addr(smem + kOffV);
             bool ok = mbar_wait_bounded(&bars.q_full, 0, a.timeout_ns, &abort_flag);
-            // Descriptors of the two stages differ by kTileBytes >> 4 in the address field.
-            constexpr uint64_t kStageStep = kTileBytes >> 4;
             const uint64_t qdesc0 = sdesc_sw128(q_base, 16, 1024);
             const uint64_t kdesc0 = sdesc_sw128(k_base, 16, 1024);
             const uint64_t vdesc0 = sdesc_sw128(v_base, kHalf, 1024);
-            auto issue_pv = [&](int t, int qt) {
-                mma_ts_k128<2048>(tmem + qt * 256 + 128, tmem + qt * 256, vdesc0 + (t & 1) * kStageStep, id_pv,
-                                  t > 0 ? 1u : 0u);
-            };
-            // The query-tile count is a compile-time constant of the issue loop: this
-            // thread is the critical path, and a runtime bound costs ~10%.
-            auto issue_all = [&](auto nq_c) {
-                constexpr int NQ = decltype(nq_c)::value;
-                for (int t = 0; ok && t < T; ++t) {
-                    const int st = t & 1;
-                    if (!mbar_test(&bars.kv_full[st], (t >> 1) & 1) &&
-                        !mbar_wait_bounded(&bars.kv_full[st], (t >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                    // TMA data is ordered by the barrier's transaction count; from t = 1
-                    // the fence after the P wait below precedes every MMA of the iteration.
-                    if (t == 0) tc_fence_after();
-                    for (int qt = 0; qt < NQ; ++qt) {
-                        if (t > 0) {
-                            if (!mbar_wait_bounded(&bars.p_full[qt], (t - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                            tc_fence_after();
-                            issue_pv(t - 1, qt);
-                        }
-                        mma_ss_k128<kHalf>(tmem + qt * 256, qdesc0 + qt * kStageStep, kdesc0 + st * kStageStep, id_qk, 0u);
-                        mma_commit(&bars.s_full[qt][st]);
-                    }
-                }
-                if (ok) {
-                    if (!mbar_wait_bounded(&bars.kv_full[T & 1], (T >> 1) & 1, a.timeout_ns, &abort_flag)) ok = false;
-                    for (int qt = 0; qt < NQ && ok; ++qt) {
-                        if (!mbar_wait_bounded(&bars.p_full[qt], (T - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
-                        tc_fence_after();
-                        issue_pv(T - 1, qt);
-                    }
-                    if (ok) mma_commit(&bars.o_full);
-                }
-            };
-            if (nq == 2) issue_all(TileCount<2>{});
-            else issue_all(TileCount<1>{});
+            if (ok)
+                ok = nq == 2 ? mma_issue_loop<2>(&bars, tmem, qdesc0, kdesc0, vdesc0, id_qk, id_pv, T, a.timeout_ns,
+                                                 &abort_flag)
+                             : mma_issue_loop<1>(&bars, tmem, qdesc0, kdesc0, vdesc0, id_qk, id_pv, T, a.timeout_ns,
+                                                 &abort_flag);
             if (!ok) {
                 fail(&abort_flag, a.status);
                 // Drain: every MMA issued so far completes before TMEM is freed.
@@ -390,35 +414,18 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
         float m_run = -INFINITY, l_run = 0.f;
         bool ok = true;
         // S row of tile t: four 32-column TMEM loads in flight, one wait, then
-        // the keys outside the row's key set set to -inf.
-        auto load_s = [&](uint32_t (&sr)[128], int t) {
+        // the keys outside the row's key set set to -inf: column c < 64 when
+        // c >= lim_a, column c >= 64 when c - 64 >= lim_b.
+        auto load_s = [&](uint32_t (&sr)[128], int lim_a, int lim_b) {
 #pragma unroll
             for (int c = 0; c < 4; ++c)
                 tmem_ld32(s_addr + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[c * 32]));
             tmem_ld_wait();
             float* s = reinterpret_cast<float*>(sr);
-            if (TOK && t < n_dt) {
-                const int lim = s_nseg - 128 * t;  // packed rows past the list are zero padding
-                if (lim < 128) {
+            if (lim_a < 64 || lim_b < 64) {
 #pragma unroll
-                    for (int c = 0; c < 128; ++c)
-                        if (c >= lim) s[c] = -INFINITY;
-                }
-            } else if (t < n_dt) {
-                const int la = seg[2 * t].y, lb = seg[2 * t + 1].y;
-                if (la < 64 || lb < 64) {
-#pragma unroll
-                    for (int c = 0; c < 128; ++c)
-                        if ((c < 64 ? c : c - 64) >= (c < 64 ? la : lb)) s[c] = -INFINITY;
-                }
-            } else {
-                const int64_t kb = W + 128ll * (t - n_dt);
-                if (kb + 127 > q0) {
-                    const int64_t lim = p - kb;  // keys kb + c with c > lim are in the future
-#pragma unroll
-                    for (int c = 0; c < 128; ++c)
-                        if (c > lim) s[c] = -INFINITY;
-                }
+                for (int c = 0; c < 128; ++c)
+                    if (c < 64 ? c >= lim_a : c - 64 >= lim_b) s[c] = -INFINITY;
             }
         };
         // p = 2^(s * scale_log2 - m) for keys [64 h, 64 h + 64): packed FMA, then
@@ -447,7 +454,25 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
             const bool got = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.s_full[qt][t & 1], (t >> 1) & 1, a.timeout_ns, &abort_flag));
             if (!got) { ok = false; break; }
             tc_fence_after();
-            float sum = 0.f;
+            // Mask limits of tile t (128: nothing masked).
+            int lim_a = 128, lim_b = 128;
+            if (TOK && t < n_dt) {
+                const int lim = s_nseg - 128 * t;  // packed rows past the list are zero padding
+                if (lim < 128) {
+                    lim_a = lim < 0 ? 0 : lim;
+                    lim_b = lim_a - 64;
+                }
+            } else if (t < n_dt) {
+                lim_a = seg[2 * t].y;
+                lim_b = seg[2 * t + 1].y;
+            } else {
+                const int64_t kb = W + 128ll * (t - n_dt);
+                if (kb + 127 > q0) {
+                    const int64_t lim = p - kb + 1;  // keys kb + c with c >= lim are in the future
+                    lim_a = lim < 0 ? 0 : (lim > 128 ? 128 : static_cast<int>(lim));
+                    lim_b = lim_a - 64;
+                }
+            }
             // Fast path: the exponentials are taken against the running max as it
             // stands, without the row max. The max only matters when the tile
             // outgrows m_run by more than the raise threshold, and the sum shows
@@ -455,68 +480,62 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
             // logit more than 9 (log2 units) above m_run. Below that every p is
             // at most 2^16, far inside the fp32 and bf16 ranges, so m_run may
             // stay; a sum that is inf or NaN fails the test as well. The first
-            // tile (m_run = -inf) and every failed tile take the exact path on a
-            // fresh copy of S (nothing has been stored over it yet).
+            // tile (m_run = -inf) and every failed tile take the exact path (row
+            // max, raise, O rescale) on a fresh copy of S: nothing has been
+            // stored over it yet.
             bool exact = !__all_sync(0xFFFFFFFFu, m_run != -INFINITY);
-            if (!exact) {
-                uint32_t sr[128];
-                load_s(sr, t);
-                const float* s = reinterpret_cast<const float*>(sr);
-                uint32_t pk[2][32];
-                const float sum0 = exp_half(s, 0, -m_run, pk[0]);
-                const float sum1 = exp_half(s, 1, -m_run, pk[1]);
-                sum = sum0 + sum1;
-                exact = __any_sync(0xFFFFFFFFu, !(sum <= kFastSumLimit));
-                if (!exact) {
-                    tmem_st32(s_addr, pk[0]);
-                    tmem_st32(s_addr + 32, pk[1]);
-                }
-            }
-            if (exact) {
-                sum = 0.f;
-                uint32_t sr[128];
-                load_s(sr, t);
-                const float* s = reinterpret_cast<const float*>(sr);
-                // Row max: eight independent three-input max chains.
-                float mx8[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) mx8[i] = s[i];
-#pragma unroll
-                for (int c = 8; c < 120; c += 16)
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) mx8[i] = fmax3(mx8[i], s[c + 2 * i], s[c + 2 * i + 1]);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[120 + i]);
-                const float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
-                                       fmaxf(mx8[6], mx8[7]));
-                const float m_new = fmaxf(m_run, mx * a.scale_log2);
-                const bool raise = m_new > m_run + kRescaleThreshold;
-                // The O rescale goes through warp-collective TMEM loads and stores,
-                // so the branch is taken by the whole warp when any row needs it;
-                // rows that do not keep their max and scale by 1.
-                if (__any_sync(0xFFFFFFFFu, raise)) {
-                    const float alpha = raise ? ex2(m_run - m_new) : 1.0f;
-                    l_run *= alpha;
-                    if (t > 0) {
+            float sum;
 #pragma unroll 1
-                        for (int c = 0; c < 8; ++c) {
-                            uint32_t v[16];
-                            tmem_ld16(o_addr + c * 16, v);
-                            tmem_ld_wait();
+            for (;;) {
+                uint32_t sr[128];
+                load_s(sr, lim_a, lim_b);
+                const float* s = reinterpret_cast<const float*>(sr);
+                if (exact) {
+                    // Row max: eight independent three-input max chains.
+                    float mx8[8];
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
-                            tmem_st16(o_addr + c * 16, v);
+                    for (int i = 0; i < 8; ++i) mx8[i] = s[i];
+#pragma unroll
+                    for (int c = 8; c < 120; c += 16)
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) mx8[i] = fmax3(mx8[i], s[c + 2 * i], s[c + 2 * i + 1]);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) mx8[i] = fmaxf(mx8[i], s[120 + i]);
+                    const float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
+                                           fmaxf(mx8[6], mx8[7]));
+                    const float m_new = fmaxf(m_run, mx * a.scale_log2);
+                    const bool raise = m_new > m_run + kRescaleThreshold;
+                    // The O rescale goes through warp-collective TMEM loads and stores,
+                    // so the branch is taken by the whole warp when any row needs it;
+                    // rows that do not keep their max and scale by 1.
+                    if (__any_sync(0xFFFFFFFFu, raise)) {
+                        const float alpha = raise ? ex2(m_run - m_new) : 1.0f;
+                        l_run *= alpha;
+                        if (t > 0) {
+#pragma unroll 1
+                            for (int c = 0; c < 8; ++c) {
+                                uint32_t v[16];
+                                tmem_ld16(o_addr + c * 16, v);
+                                tmem_ld_wait();
+#pragma unroll
+                                for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+                                tmem_st16(o_addr + c * 16, v);
+                            }
                         }
+                        if (raise) m_run = m_new;
                     }
-                    if (raise) m_run = m_new;
                 }
                 const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    uint32_t pk[32];
-                    sum += exp_half(s, h, neg_m, pk);
-                    tmem_st32(s_addr + h * 32, pk);
+                uint32_t pk[2][32];
+                sum = exp_half(s, 0, neg_m, pk[0]);
+                sum += exp_half(s, 1, neg_m, pk[1]);
+                if (!exact && __any_sync(0xFFFFFFFFu, !(sum <= kFastSumLimit))) {
+                    exact = true;
+                    continue;
                 }
+                tmem_st32(s_addr, pk[0]);
+                tmem_st32(s_addr + 32, pk[1]);
+                break;
             }
             l_run += sum;
             tmem_st_wait();
