@@ -181,21 +181,24 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     // ---- work item: a 128-row query block of one sub-chunk and a pair of
     // query heads. The grid holds exactly the blocks of the sub-chunks in
     // range (no idle CTAs whatever the clustering), outer chunk by outer
-    // chunk, so one cluster's distant K/V set is live in L2 at a time; within
-    // a chunk the last block comes first, which issues each cluster's
-    // heaviest rows (longest window) first. ----
-    int lin = blockIdx.x;
-    const int hp = lin % (a.Hkv * a.pairs);
-    lin /= a.Hkv * a.pairs;
-    const int kvh = hp / a.pairs;
-    const int h0 = kvh * a.g + 2 * (hp % a.pairs);
-    const int nq = (h0 + 1 < (kvh + 1) * a.g) ? 2 : 1;  // query tiles (heads) of this CTA
-    const int per_chunk = a.sc_per_chunk * a.qb_per_sc;
-    const int c = lin / per_chunk;
+    // chunk, and within a chunk KV head by KV head, so the CTAs resident at
+    // a time share the K/V rows of one or two KV heads of one cluster (a few
+    // MB, which L2 keeps); for each KV head the chunk's last query block
+    // comes first, which issues the heaviest rows (longest window) first. ----
+    const int per_chunk = a.sc_per_chunk * a.qb_per_sc;  // query blocks of a full chunk
+    const int per_chunk_ctas = per_chunk * a.Hkv * a.pairs;
+    const int c = static_cast<int>(blockIdx.x) / per_chunk_ctas;
     const int sc0 = a.sc_begin + c * a.sc_per_chunk;
     const int n_sc = (a.sc_end - sc0 < a.sc_per_chunk) ? a.sc_end - sc0 : a.sc_per_chunk;
-    const int idx = n_sc * a.qb_per_sc - 1 - (lin - c * per_chunk);
-    if (idx < 0) return;
+    const int n_qb = n_sc * a.qb_per_sc;  // query blocks of this chunk
+    int rem = static_cast<int>(blockIdx.x) - c * per_chunk_ctas;
+    const int kvh = rem / (n_qb * a.pairs);
+    rem -= kvh * n_qb * a.pairs;
+    const int qb = rem / a.pairs;
+    const int h0 = kvh * a.g + 2 * (rem - qb * a.pairs);
+    const int nq = (h0 + 1 < (kvh + 1) * a.g) ? 2 : 1;  // query tiles (heads) of this CTA
+    const int idx = n_qb - 1 - qb;
+    if (idx < 0 || kvh >= a.Hkv) return;
     const int sc = sc0 + idx / a.qb_per_sc;
     const int u = unit_of_subchunk(a.ut, sc);
     int anchor;
