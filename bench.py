@@ -47,6 +47,10 @@ def parse_args():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--mode", choices=["cluster", "subchunk"], default="cluster")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--selection-check", action="store_true",
+                    help="without the CPU baseline: still compare the GPU selection with the oracle's steps (a)-(c)")
+    ap.add_argument("--no-other-configs", action="store_true",
+                    help="skip the side runs of the other workload configs after the headline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-full", action="store_true",
                     help="skip timing the oracle over every row of the 4K and 32K layers")
@@ -347,6 +351,58 @@ def loop_calls(w, mode_sub: bool):
     return out
 
 
+# The other workload configs, each run after the headline as its own process
+# (Algorithm 2 loop in both modes, plus the whole-sequence launches), with the
+# GPU selection compared with the oracle's where steps (a)-(c) fit in seconds.
+OTHER_CONFIGS = (("gqa4-4k", True), ("llama8b-32k", True), ("llama8b-64k-32l", False), ("llama8b-1m", True),
+                 ("llama8b-128k-tok", True))
+OTHER_STEPS, OTHER_WARMUP = 3, 3
+
+
+def other_configs() -> dict:
+    """Side runs of the other configs: per workload the SCR and per-sub-chunk
+    loops (TTFT of one layer, or of the stack), attention throughput, selection
+    time and retrieval calls, and the selection agreement with the oracle."""
+    import subprocess
+
+    out = {}
+    for name, check in OTHER_CONFIGS:
+        cmd = [sys.executable, os.path.abspath(__file__), "--workload", name, "--steps", str(OTHER_STEPS),
+               "--warmup", str(OTHER_WARMUP), "--no-e2e", "--no-cpu-baseline", "--no-other-configs"]
+        if check:
+            cmd.append("--selection-check")
+        t0 = time.perf_counter()
+        r = subprocess.run(cmd, capture_output=True, text=True, cwd=ROOT)
+        wall = time.perf_counter() - t0
+        lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+        if r.returncode != 0 or not lines:
+            out[name] = {"error": (r.stderr.strip().splitlines() or ["no output"])[-1][:300], "rc": r.returncode}
+            continue
+        d = json.loads(lines[-1])
+        o = d.get("other_mode", {})
+        rec = {
+            "n_tokens": d["config"]["n_tokens"], "layers": d["config"].get("layers", 1),
+            "steps": d["steps"], "warmup": d["warmup"], "wall_s": round(wall, 1),
+            "cluster": {"ttft_ms": d["ms_per_step"], "tokens_per_s": d["value"],
+                        "attention_tflops": d["roofline"]["achieved"], "attention_frac": d["roofline"]["frac"],
+                        "select_ms": d.get("stages_ms", {}).get("select"),
+                        "retrieval_calls": d["retrieval_calls"], "units": d["units"],
+                        "batched_ms": d.get("batched", {}).get("ms_per_step")},
+            "subchunk": {"ttft_ms": o.get("ms_per_step"), "tokens_per_s": o.get("tokens_per_s"),
+                         "attention_tflops": o.get("attn_tflops"),
+                         "select_ms": o.get("stages_ms", {}).get("select"),
+                         "retrieval_calls": o.get("retrieval_calls"), "units": o.get("units"),
+                         "batched_ms": o.get("batched", {}).get("ms_per_step")},
+            "scr_over_subchunk": d.get("scr_over_subchunk"), "attn_flops_ratio": d.get("attn_flops_ratio"),
+            "clocks": d.get("clocks"),
+        }
+        if "selection_match_units" in d:
+            rec["selection"] = {k: d[k] for k in ("selection_match_units", "near_tie_units",
+                                                  "selection_mismatch_units")}
+        out[name] = rec
+    return out
+
+
 def run_scale(args):
     import torch
 
@@ -597,6 +653,14 @@ def run_scale(args):
                        "api": "scale_prefill_host (pinned host buffers; pieces of outer chunks, copies "
                               "overlapped with the compute)"}
         del arena
+
+    if rank == 0 and world == 1 and args.no_cpu_baseline and args.selection_check:
+        import oracle
+
+        line.update(selection_agreement(w, oracle.run_path(w, q, k, v, per_subchunk=per_sub), sel_gpu, cnt_gpu))
+
+    if rank == 0 and world == 1 and not args.no_other_configs and w.name == DEFAULT_WORKLOAD and not args.paged:
+        line["other_configs"] = other_configs()
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         r = oracle_sample(w, q, k, v, per_sub)

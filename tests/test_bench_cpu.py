@@ -73,3 +73,46 @@ def test_launch_counts():
     assert bench.launches(workload("llama8b-32k", block_size=1, top_k=1024))["total"] == 3 + 5 + 3
     assert bench.launches(workload("llama8b-64k-32l"), 8)["total"] == 4 + 8 * 5
     assert bench.launches(workload("llama8b-64k-32l"), 8, 8)["total"] == 8 * 4 + 8 * 5  # per-chunk step (a)
+
+
+def test_other_configs_compacts_each_side_run(monkeypatch):
+    """The side runs of the other configs: one process per workload; a layer's
+    line (with both modes and the selection check) and a stack's line (no
+    batched form) are compacted, a failed run is reported, not raised."""
+    import subprocess
+
+    layer = {"config": {"n_tokens": 32768}, "steps": 3, "warmup": 3, "ms_per_step": 6.0, "value": 5.4e6,
+             "roofline": {"achieved": 1500.0, "frac": 0.78}, "stages_ms": {"select": 1.1},
+             "retrieval_calls": 3, "units": 4, "batched": {"ms_per_step": 2.7},
+             "other_mode": {"ms_per_step": 5.0, "tokens_per_s": 6.5e6, "attn_tflops": 1300.0,
+                            "stages_ms": {"select": 3.0}, "retrieval_calls": 30, "units": 32,
+                            "batched": {"ms_per_step": 2.0}},
+             "scr_over_subchunk": 1.2, "attn_flops_ratio": 1.5, "clocks": {"sm_mhz": 2000.0},
+             "selection_match_units": 4, "near_tie_units": 0, "selection_mismatch_units": 0}
+    stack = {"config": {"n_tokens": 65536, "layers": 32}, "steps": 3, "warmup": 3, "ms_per_step": 200.0,
+             "value": 3.3e5, "roofline": {"achieved": 1600.0, "frac": 0.83}, "retrieval_calls": 224,
+             "units": 256, "other_mode": {"ms_per_step": 230.0, "tokens_per_s": 2.8e5, "attn_tflops": 1400.0,
+                                          "retrieval_calls": 1984, "units": 2048},
+             "scr_over_subchunk": 0.87, "attn_flops_ratio": 1.58, "clocks": None}
+    calls = []
+
+    def fake_run(cmd, **kw):
+        name = cmd[cmd.index("--workload") + 1]
+        calls.append(cmd)
+        if name == "llama8b-1m":
+            return subprocess.CompletedProcess(cmd, 1, "", "RuntimeError: boom\n")
+        out = stack if name == "llama8b-64k-32l" else layer
+        return subprocess.CompletedProcess(cmd, 0, "log line\n" + json.dumps(out) + "\n", "")
+
+    monkeypatch.setattr(subprocess, "run", fake_run)
+    got = bench.other_configs()
+    assert [c[c.index("--workload") + 1] for c in calls] == [n for n, _ in bench.OTHER_CONFIGS]
+    assert all("--no-other-configs" in c for c in calls)
+    assert ("--selection-check" in calls[2]) is False  # the stack runs no oracle check
+    l32 = got["llama8b-32k"]
+    assert l32["cluster"]["ttft_ms"] == 6.0 and l32["subchunk"]["ttft_ms"] == 5.0
+    assert l32["cluster"]["batched_ms"] == 2.7 and l32["subchunk"]["select_ms"] == 3.0
+    assert l32["selection"]["selection_mismatch_units"] == 0
+    st = got["llama8b-64k-32l"]
+    assert st["layers"] == 32 and st["cluster"]["batched_ms"] is None and "selection" not in st
+    assert got["llama8b-1m"] == {"error": "RuntimeError: boom", "rc": 1}
