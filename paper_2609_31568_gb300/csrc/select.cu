@@ -232,11 +232,27 @@ __global__ void __launch_bounds__(256) k_stats(SelArgs a, const float* __restric
     cand_range(a, s, &lo, &hi);
     if (lo >= hi) return;
     const float* z = logits + (static_cast<int64_t>(u) * a.Hq + h) * a.nb;
+    // Eight loads in flight per lane; each lane still combines its values in
+    // index order, so the result does not depend on the batching.
+    constexpr int kIn = 8;
     float m = -INFINITY;
-    for (int64_t b = lo + lane; b < hi; b += 32) m = fmaxf(m, z[b]);
+    for (int64_t b0 = lo + lane; b0 < hi; b0 += 32 * kIn) {
+        float x[kIn];
+#pragma unroll
+        for (int i = 0; i < kIn; ++i) x[i] = b0 + 32 * i < hi ? z[b0 + 32 * i] : -INFINITY;
+#pragma unroll
+        for (int i = 0; i < kIn; ++i) m = fmaxf(m, x[i]);
+    }
     for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
     float sum = 0.f;
-    for (int64_t b = lo + lane; b < hi; b += 32) sum += expf(z[b] - m);
+    for (int64_t b0 = lo + lane; b0 < hi; b0 += 32 * kIn) {
+        float x[kIn];
+#pragma unroll
+        for (int i = 0; i < kIn; ++i) x[i] = b0 + 32 * i < hi ? z[b0 + 32 * i] : 0.f;
+#pragma unroll
+        for (int i = 0; i < kIn; ++i)
+            if (b0 + 32 * i < hi) sum += expf(x[i] - m);
+    }
     for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
     if (lane == 0) {
         stats[(static_cast<int64_t>(u) * a.Hq + h) * 2] = m;
@@ -262,9 +278,22 @@ __global__ void __launch_bounds__(256) k_vote(SelArgs a, const float* __restrict
     float score = __int_as_float(0x7FC00000);
     if (b >= lo && b < hi) {
         score = 0.f;
-        for (int h = 0; h < a.Hq; ++h) {
-            const int64_t uh = static_cast<int64_t>(u) * a.Hq + h;
-            score += expf(logits[uh * a.nb + b] - stats[uh * 2]) * stats[uh * 2 + 1];
+        const float* zb = logits + static_cast<int64_t>(u) * a.Hq * a.nb + b;
+        const float* sb = stats + static_cast<int64_t>(u) * a.Hq * 2;
+        // Eight heads' loads in flight at a time, added in head order.
+        constexpr int kIn = 8;
+        for (int h0 = 0; h0 < a.Hq; h0 += kIn) {
+            float z[kIn], mx[kIn], inv[kIn];
+#pragma unroll
+            for (int i = 0; i < kIn; ++i) {
+                const int h = h0 + i < a.Hq ? h0 + i : a.Hq - 1;
+                z[i] = zb[static_cast<int64_t>(h) * a.nb];
+                mx[i] = sb[2 * h];
+                inv[i] = sb[2 * h + 1];
+            }
+#pragma unroll
+            for (int i = 0; i < kIn; ++i)
+                if (h0 + i < a.Hq) score += expf(z[i] - mx[i]) * inv[i];
         }
     }
     scores[static_cast<int64_t>(u) * a.nb + b] = score;
