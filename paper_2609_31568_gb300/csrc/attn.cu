@@ -580,41 +580,77 @@ k_sparse_attn(const __grid_constant__ CUtensorMap tq, const __grid_constant__ CU
     }
 }
 
-// Block size 1, step 1 of 2: the distant list of every unit, one warp per
+// Block size 1, step 1 of 2: the distant list of every unit, one CTA per
 // unit: the sinks [0, min(n_sink, W_u)), then every selected token in
 // [n_sink, W_u) larger than the entry before it (each key once, ascending).
-__global__ void __launch_bounds__(32) k_tok_lists(Units ut, int sc_begin, int sc_end, int n_sink, int n_local,
-                                                  int k, const int32_t* __restrict__ sel,
-                                                  const int32_t* __restrict__ sel_count,
-                                                  int32_t* __restrict__ list, int32_t* __restrict__ count, int slots)
+// The selected entries are compacted in order by one block-wide scan: each
+// thread takes kListPer consecutive entries.
+constexpr int kListThreads = 1024;
+constexpr int kListPer = 8;
+__global__ void __launch_bounds__(kListThreads) k_tok_lists(Units ut, int sc_begin, int sc_end, int n_sink,
+                                                            int n_local, int k, const int32_t* __restrict__ sel,
+                                                            const int32_t* __restrict__ sel_count,
+                                                            int32_t* __restrict__ list, int32_t* __restrict__ count,
+                                                            int slots)
 {
+    __shared__ int s_warp[kListThreads / 32];
     const int u = unit_lower_bound(ut, sc_begin) + static_cast<int>(blockIdx.x);
     if (u >= unit_lower_bound(ut, sc_end)) return;
-    const int lane = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     int anchor;
     int64_t s_u, e_u;
     unit_range(ut, u, &anchor, &s_u, &e_u);
     const int64_t W = (s_u - n_local > 0) ? s_u - n_local : 0;
     int32_t* out = list + static_cast<int64_t>(u) * slots;
     const int n_s = static_cast<int>(n_sink < W ? n_sink : W);
-    for (int i = lane; i < n_s; i += 32) out[i] = i;
-    int base = n_s;
+    for (int i = tid; i < n_s; i += kListThreads) out[i] = i;
     int cnt = sel_count[u];
     cnt = cnt < 0 ? 0 : (cnt > k ? k : cnt);
     const int32_t* sl = sel + static_cast<int64_t>(u) * k;
-    for (int c0 = 0; c0 < cnt; c0 += 32) {
-        const int i = c0 + lane;
-        bool valid = false;
-        int32_t tok = 0;
-        if (i < cnt) {
-            tok = sl[i];
-            valid = tok >= n_sink && tok < W && (i == 0 || tok > sl[i - 1]);
+    int base = n_s;
+    for (int c0 = 0; c0 < cnt; c0 += kListThreads * kListPer) {
+        const int i0 = c0 + tid * kListPer;
+        int32_t tok[kListPer];
+        int prev = (i0 > 0 && i0 - 1 < cnt) ? sl[i0 - 1] : -1;
+        unsigned valid = 0u;
+#pragma unroll
+        for (int j = 0; j < kListPer; ++j) {
+            const int i = i0 + j;
+            tok[j] = i < cnt ? sl[i] : -1;
+            if (i < cnt && tok[j] >= n_sink && tok[j] < W && tok[j] > prev) valid |= 1u << j;
+            if (i < cnt) prev = tok[j];
         }
-        const uint32_t b = __ballot_sync(0xFFFFFFFFu, valid);
-        if (valid) out[base + __popc(b & ((1u << lane) - 1u))] = tok;
-        base += __popc(b);
+        const int mine = __popc(valid);
+        int incl = mine;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        if (lane == 31) s_warp[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            const int x = s_warp[lane];
+            int xi = x;
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(0xFFFFFFFFu, xi, o);
+                if (lane >= o) xi += y;
+            }
+            s_warp[lane] = xi - x;  // exclusive prefix of the warps
+        }
+        __syncthreads();
+        int pos = base + s_warp[warp] + incl - mine;
+#pragma unroll
+        for (int j = 0; j < kListPer; ++j)
+            if ((valid >> j) & 1u) out[pos++] = tok[j];
+        const int total = __shfl_sync(0xFFFFFFFFu, incl, 31);
+        __syncthreads();
+        // the block total: the last warp's exclusive prefix plus its total
+        if (tid == kListThreads - 1) s_warp[0] = s_warp[warp] + total;
+        __syncthreads();
+        base += s_warp[0];
+        __syncthreads();
     }
-    if (lane == 0) count[u] = base;
+    if (tid == 0) count[u] = base;
 }
 
 // Block size 1, step 2 of 2: copy the listed K and V rows of unit u
@@ -740,7 +776,7 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
     if (tok) {
         int32_t* list = reinterpret_cast<int32_t*>(ws + lay.tok_list);
         int32_t* cnt = const_cast<int32_t*>(a.tok_count);
-        k_tok_lists<<<a.n_sc, 32, 0, st>>>(a.ut, a.sc_begin, a.sc_end, d.n_sink, d.n_local, d.k, sel_blocks,
+        k_tok_lists<<<a.n_sc, kListThreads, 0, st>>>(a.ut, a.sc_begin, a.sc_end, d.n_sink, d.n_local, d.k, sel_blocks,
                                            sel_count, list, cnt, slots);
         k_tok_pack<<<dim3(a.n_sc, d.Hkv, (slots + kPackSlots - 1) / kPackSlots), 256, 0, st>>>(
             a.ut, a.sc_begin, a.sc_end, d.Hkv, pg, list, cnt, static_cast<const uint4*>(k),
