@@ -25,6 +25,9 @@
 //                   owns its (unit, token) cells, so no atomics are needed.
 //
 // Each CTA owns a tile of 128 / g units and a range of 128 g tokens (<= 1024).
+// Calls of at most 16 units (every call of the Algorithm 2 loop) use
+// k_tok_score_s instead: 16 (unit, head) columns per tile, tokens as the MMA
+// rows and the three parts side by side in one N = 48 operand.
 // Warp 0 lane 0 issues TMA loads (the fingerprint parts of one KV head, then
 // 128-token key tiles into a 2-stage ring), warp 1 lane 0 issues the MMAs
 // (TMEM: two 128-column accumulators), warps 2-5 run the epilogue. Every wait
@@ -343,6 +346,311 @@ k_tok_score(const __grid_constant__ CUtensorMap tf, const __grid_constant__ CUte
     }
 }
 
+// ---- the same two passes for calls with few units (every call of the
+// Algorithm 2 loop covers one cluster or one sub-chunk): a unit tile of
+// 16 / G units, i.e. 16 (unit, head) columns. The 128 tokens of a key tile
+// are the MMA rows and the three bf16 parts of the 16 fingerprint columns sit
+// side by side in one N = 48 operand (part s at columns [16 s, 16 s + 16)),
+// so one MMA per K-step yields the three partial dot products: 8 MMAs per key
+// tile instead of 24, and a 12 KB fingerprint tile per KV head instead of
+// 96 KB. Pass 0 keeps a running (max, sum) per column in each token's thread
+// and merges the 128 threads once per KV head (a fixed shuffle tree, then
+// the four warps in order); pass 1 keeps each token's votes in registers.
+constexpr int kNc = 16;                        // (unit, head) columns of a small tile
+constexpr uint32_t kFsHalf = 3 * kNc * 128;    // one 64-column half of the 48-row operand: 6 KB
+constexpr uint32_t kOffFs = 0;                 // fingerprint parts, 12 KB
+constexpr uint32_t kOffKs = 2 * kFsHalf;       // 2 key stages (a multiple of 1024)
+constexpr uint32_t kSmemTokS = kOffKs + 2 * kTile + 1024;
+static_assert(kOffKs % 1024 == 0, "key stages must stay 1024-aligned");
+
+// (m, s) of a sum of 2^(z - m) terms merged with another: both in log2 units.
+__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2)
+{
+    const float mn = fmaxf(m, m2);
+    if (mn == -INFINITY) return;
+    s = s * ex2(m - mn) + s2 * ex2(m2 - mn);
+    m = mn;
+}
+
+template <int PASS, int G>
+__global__ void __launch_bounds__(kTokThreads, 2)
+k_tok_score_s(const __grid_constant__ CUtensorMap tfs, const __grid_constant__ CUtensorMap tk, const TokArgs a)
+{
+    constexpr int US = kNc / G;  // units of the tile
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ TokBars bars;
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+    __shared__ int s_W[US];
+    __shared__ float2 s_col[kNc];
+    __shared__ float2 s_red[4][kNc];
+
+    const int u_first = unit_lower_bound(a.ut, a.sc_begin);
+    const int u_end = unit_lower_bound(a.ut, a.sc_end);
+    const int u0 = u_first + static_cast<int>(blockIdx.y) * US;
+    if (u0 >= u_end) return;
+    const int n_u = (u_end - u0 < US) ? u_end - u0 : US;
+    const int x = blockIdx.x;
+    const int r0 = x * a.range;
+    const int r1 = (r0 + a.range < a.N) ? r0 + a.range : a.N;
+    const int64_t w_max = window_start(a, u0 + n_u - 1);
+    const int c_hi = static_cast<int>(w_max < r1 ? w_max : r1);
+    const bool work = c_hi > r0 && c_hi > a.n_sink;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    if (!work) {
+        if (PASS == 1) {  // no candidate in the range: every score is NaN
+            for (int ul = 0; ul < n_u; ++ul)
+                for (int t = r0 + tid; t < r1; t += blockDim.x)
+                    a.scores[static_cast<int64_t>(u0 + ul) * a.N + t] = __int_as_float(0x7FC00000);
+        }
+        return;
+    }
+    const int n_tiles = (c_hi - r0 + 127) / 128;
+
+    uint8_t* smem = smem_raw + ((1024u - (smem_addr(smem_raw) & 1023u)) & 1023u);
+    if (tid < US) s_W[tid] = (tid < n_u) ? static_cast<int>(window_start(a, u0 + tid)) : 0;
+    if (tid == 0) {
+        abort_flag = 0;
+        mbar_init(&bars.f_full, 1);
+        mbar_init(&bars.f_empty, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&bars.k_full[i], 1);
+            mbar_init(&bars.k_empty[i], 1);
+            mbar_init(&bars.d_full[i], 1);
+            mbar_init(&bars.d_empty[i], 128);
+        }
+        mbar_init(&bars.drain, 1);
+        fence_barrier_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_slot, 128);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            tma_prefetch_desc(&tfs);
+            tma_prefetch_desc(&tk);
+            int gt = 0;
+            int issued_k0 = 0, issued_k1 = 0, issued_f = 0;
+            for (int j = 0; j < a.Hkv && !abort_flag; ++j) {
+                if (j > 0 && !mbar_wait_bounded(&bars.f_empty, (j - 1) & 1, a.timeout_ns, &abort_flag)) {
+                    tok_fail(&abort_flag, a.status);
+                    break;
+                }
+                mbar_arrive_expect_tx(&bars.f_full, 2 * kFsHalf);
+                ++issued_f;
+                for (int sp = 0; sp < 3; ++sp)
+                    for (int hf = 0; hf < 2; ++hf)
+                        tma_load_4d(smem + kOffFs + hf * kFsHalf + sp * kNc * 128, &tfs, &bars.f_full, hf * 64,
+                                    u0 * G, j, sp);
+                for (int i = 0; i < n_tiles; ++i, ++gt) {
+                    const int st = gt & 1;
+                    if (gt >= 2 && !mbar_wait_bounded(&bars.k_empty[st], ((gt >> 1) - 1) & 1, a.timeout_ns, &abort_flag)) {
+                        tok_fail(&abort_flag, a.status);
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&bars.k_full[st], kTile);
+                    if (st) ++issued_k1; else ++issued_k0;
+                    const int32_t ra = kv_row_tma(a.pg, r0 + 128 * i);
+                    const int32_t rb = kv_row_tma(a.pg, r0 + 128 * i + 64);
+                    for (int hf = 0; hf < 2; ++hf) {
+                        uint8_t* dst = smem + kOffKs + st * kTile + hf * kHalfT;
+                        tma_load_3d(dst, &tk, &bars.k_full[st], hf * 64, j, ra);
+                        tma_load_3d(dst + kHalfT / 2, &tk, &bars.k_full[st], hf * 64, j, rb);
+                    }
+                }
+            }
+            if (abort_flag) {
+                if (issued_f) mbar_wait_bounded(&bars.f_full, (issued_f - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_k0) mbar_wait_bounded(&bars.k_full[0], (issued_k0 - 1) & 1, a.timeout_ns, nullptr);
+                if (issued_k1) mbar_wait_bounded(&bars.k_full[1], (issued_k1 - 1) & 1, a.timeout_ns, nullptr);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, 3 * kNc, 0);
+            const uint64_t fdesc = sdesc_sw128(smem_addr(smem + kOffFs), 16, 1024);
+            const uint64_t kdesc0 = sdesc_sw128(smem_addr(smem + kOffKs), 16, 1024);
+            constexpr uint64_t kStep = kTile >> 4;
+            bool ok = true;
+            int gt = 0;
+            for (int j = 0; ok && j < a.Hkv; ++j) {
+                if (!mbar_wait_bounded(&bars.f_full, j & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                for (int i = 0; i < n_tiles; ++i, ++gt) {
+                    const int st = gt & 1;
+                    if (!mbar_wait_bounded(&bars.k_full[st], (gt >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                    if (gt >= 2 && !mbar_wait_bounded(&bars.d_empty[st], ((gt >> 1) - 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+                    tc_fence_after();
+                    // rows: the tile's 128 tokens (A = keys), columns: 3 parts x 16
+                    mma_ss_k128_ab<kHalfT, kFsHalf>(tmem + st * 64, kdesc0 + st * kStep, fdesc, idesc, 0u);
+                    mma_commit(&bars.d_full[st]);
+                    mma_commit(&bars.k_empty[st]);
+                }
+                if (ok) mma_commit(&bars.f_empty);
+            }
+            if (!ok) {
+                tok_fail(&abort_flag, a.status);
+                mma_commit(&bars.drain);
+                mbar_wait_bounded(&bars.drain, 0, a.timeout_ns, nullptr);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int q = warp & 3;  // TMEM lane quarter this warp may access
+        const int r = q * 32 + lane;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(q * 32) << 16);
+        bool ok = true;
+        int gt = 0;
+        // z of this thread's token for the 16 columns: the three parts added
+        auto load_z = [&](int st, float (&z)[kNc]) {
+            uint32_t p0[16], p1[16], p2[16];
+            tmem_ld16(lane_base + st * 64, p0);
+            tmem_ld16(lane_base + st * 64 + kNc, p1);
+            tmem_ld16(lane_base + st * 64 + 2 * kNc, p2);
+            tmem_ld_wait();
+#pragma unroll
+            for (int c = 0; c < kNc; ++c)
+                z[c] = (__uint_as_float(p0[c]) + __uint_as_float(p1[c])) + __uint_as_float(p2[c]);
+        };
+        if (PASS == 0) {
+            for (int j = 0; j < a.Hkv; ++j) {
+                float m[kNc], sm[kNc];
+#pragma unroll
+                for (int c = 0; c < kNc; ++c) {
+                    m[c] = -INFINITY;
+                    sm[c] = 0.f;
+                }
+                for (int i = 0; i < n_tiles; ++i, ++gt) {
+                    const int st = gt & 1;
+                    if (!ok) continue;
+                    const bool got = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.d_full[st], (gt >> 1) & 1, a.timeout_ns, &abort_flag));
+                    if (!got) { ok = false; continue; }
+                    tc_fence_after();
+                    float z[kNc];
+                    load_z(st, z);
+                    tc_fence_before();
+                    mbar_arrive(&bars.d_empty[st]);
+                    const int t = r0 + 128 * i + r;
+                    if (t < a.n_sink || t >= c_hi) continue;
+#pragma unroll
+                    for (int c = 0; c < kNc; ++c) {
+                        const int ul = c / G;
+                        if (ul < n_u && t < s_W[ul]) {
+                            const float zz = z[c] * a.scale2;
+                            const float mn = fmaxf(m[c], zz);
+                            sm[c] = sm[c] * ex2(m[c] - mn) + ex2(zz - mn);
+                            m[c] = mn;
+                        }
+                    }
+                }
+                // merge the 128 tokens' (max, sum) per column: lanes, then warps in order
+#pragma unroll
+                for (int c = 0; c < kNc; ++c)
+                    for (int o = 16; o > 0; o >>= 1) {
+                        const float m2 = __shfl_xor_sync(0xFFFFFFFFu, m[c], o);
+                        const float s2 = __shfl_xor_sync(0xFFFFFFFFu, sm[c], o);
+                        lse_merge(m[c], sm[c], m2, s2);
+                    }
+                if (lane < kNc) {
+                    float mv = m[0], sv = sm[0];
+#pragma unroll
+                    for (int c = 1; c < kNc; ++c)
+                        if (lane == c) {
+                            mv = m[c];
+                            sv = sm[c];
+                        }
+                    s_red[q][lane] = make_float2(mv, sv);
+                }
+                named_barrier(1, 128);
+                if (r < kNc && ok) {
+                    const int ul = r / G, hl = r % G;
+                    float mv = s_red[0][r].x, sv = s_red[0][r].y;
+                    for (int w = 1; w < 4; ++w) lse_merge(mv, sv, s_red[w][r].x, s_red[w][r].y);
+                    if (ul < n_u)
+                        a.part[(static_cast<int64_t>(u0 + ul) * a.Hq + j * G + hl) * a.n_ranges + x] =
+                            make_float2(mv, sv);
+                }
+                named_barrier(1, 128);
+            }
+        } else {
+            // votes of this thread's token in each key tile of the range, per unit
+            constexpr int kTiles = G <= 8 ? G : 8;  // a.range / 128
+            float vote[kTiles][US];
+#pragma unroll
+            for (int i = 0; i < kTiles; ++i)
+#pragma unroll
+                for (int ul = 0; ul < US; ++ul) vote[i][ul] = 0.f;
+            for (int j = 0; j < a.Hkv; ++j) {
+                named_barrier(1, 128);
+                if (r < kNc) {
+                    const int ul = r / G, hl = r % G;
+                    s_col[r] = (ul < n_u) ? a.stats[static_cast<int64_t>(u0 + ul) * a.Hq + j * G + hl]
+                                          : make_float2(0.f, 0.f);
+                }
+                named_barrier(1, 128);
+#pragma unroll
+                for (int i = 0; i < kTiles; ++i) {
+                    if (i >= n_tiles) continue;
+                    const int st = gt & 1;
+                    const int ph = (gt >> 1) & 1;
+                    ++gt;
+                    if (!ok) continue;
+                    const bool got = __all_sync(0xFFFFFFFFu, mbar_wait_bounded(&bars.d_full[st], ph, a.timeout_ns, &abort_flag));
+                    if (!got) { ok = false; continue; }
+                    tc_fence_after();
+                    float z[kNc];
+                    load_z(st, z);
+                    tc_fence_before();
+                    mbar_arrive(&bars.d_empty[st]);
+                    const int t = r0 + 128 * i + r;
+                    if (t < a.n_sink || t >= c_hi) continue;
+#pragma unroll
+                    for (int ul = 0; ul < US; ++ul) {
+                        float acc = 0.f;
+#pragma unroll
+                        for (int hl = 0; hl < G; ++hl) {
+                            const int c = ul * G + hl;
+                            const float2 cs = s_col[c];
+                            acc += ex2(z[c] * a.scale2 - cs.x) * cs.y;
+                        }
+                        if (ul < n_u && t < s_W[ul]) vote[i][ul] += acc;
+                    }
+                }
+            }
+            if (__all_sync(0xFFFFFFFFu, ok && !abort_flag)) {
+#pragma unroll
+                for (int i = 0; i < kTiles; ++i) {
+                    const int t = r0 + 128 * i + r;
+                    if (t >= r1) continue;
+#pragma unroll
+                    for (int ul = 0; ul < US; ++ul)
+                        if (ul < n_u)
+                            a.scores[static_cast<int64_t>(u0 + ul) * a.N + t] =
+                                (t >= a.n_sink && t < s_W[ul]) ? vote[i][ul] : __int_as_float(0x7FC00000);
+                }
+            } else {
+                ok = false;
+            }
+        }
+        if (!ok) tok_fail(&abort_flag, a.status);
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 128);
+    }
+}
+
 // v_a(u)^(h) (fp32) -> three bf16 parts; row (u, h) of KV head j = h / g at
 // [part][j][u][h % g][128].
 __global__ void __launch_bounds__(128) k_tok_split(TokArgs a, const float* __restrict__ fp,
@@ -416,6 +724,26 @@ cudaError_t run_tok_passes(dim3 grid, int64_t rows, const CUtensorMap& tf, const
     return cudaGetLastError();
 }
 
+// The two passes with small unit tiles (k_tok_score_s): calls of at most
+// kSmallUnits units.
+constexpr int kSmallUnits = 16;
+
+template <int G>
+cudaError_t run_tok_passes_s(dim3 grid, int64_t rows, const CUtensorMap& tfs, const CUtensorMap& tk,
+                             const TokArgs& a, cudaStream_t st)
+{
+    cudaError_t e = cudaFuncSetAttribute(k_tok_score_s<0, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kSmemTokS));
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_tok_score_s<1, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kSmemTokS));
+    if (e != cudaSuccess) return e;
+    k_tok_score_s<0, G><<<grid, kTokThreads, kSmemTokS, st>>>(tfs, tk, a);
+    k_tok_merge<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a);
+    k_tok_score_s<1, G><<<grid, kTokThreads, kSmemTokS, st>>>(tfs, tk, a);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 int tok_range(const Derived& d)
@@ -463,10 +791,35 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
         return cudaErrorInvalidValue;
 
     k_tok_split<<<static_cast<unsigned>(max_units) * d.Hq, 128, 0, st>>>(a, fingerprints, parts, static_cast<int>(d.M));
-    const int tiles_u = (max_units + a.U - 1) / a.U;
-    const dim3 grid(static_cast<unsigned>(a.n_ranges), static_cast<unsigned>(tiles_u));
     const int64_t rows = static_cast<int64_t>(max_units) * d.Hq;
     cudaError_t e = cudaSuccess;
+    if (max_units <= kSmallUnits) {
+        // few units (every call of the Algorithm 2 loop): 16 (unit, head) columns per tile
+        CUtensorMap tfs;
+        const uint32_t fbox_s[4] = {64, kNc, 1, 1};
+        if (!scale_host::make_dense_bf16_map(&tfs, parts, 4, fdims, fbox_s)) return cudaErrorInvalidValue;
+        const int us = kNc / d.g;
+        const dim3 grid_s(static_cast<unsigned>(a.n_ranges), static_cast<unsigned>((max_units + us - 1) / us));
+        switch (d.g) {
+        case 1: e = run_tok_passes_s<1>(grid_s, rows, tfs, tk, a, st); break;
+        case 2: e = run_tok_passes_s<2>(grid_s, rows, tfs, tk, a, st); break;
+        case 3: e = run_tok_passes_s<3>(grid_s, rows, tfs, tk, a, st); break;
+        case 4: e = run_tok_passes_s<4>(grid_s, rows, tfs, tk, a, st); break;
+        case 5: e = run_tok_passes_s<5>(grid_s, rows, tfs, tk, a, st); break;
+        case 6: e = run_tok_passes_s<6>(grid_s, rows, tfs, tk, a, st); break;
+        case 7: e = run_tok_passes_s<7>(grid_s, rows, tfs, tk, a, st); break;
+        case 8: e = run_tok_passes_s<8>(grid_s, rows, tfs, tk, a, st); break;
+        default: return cudaErrorInvalidValue;
+        }
+        if (e == cudaSuccess) e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        const TopkScratch scratch{reinterpret_cast<int32_t*>(ws + lay.topk_hist),
+                                  reinterpret_cast<int32_t*>(ws + lay.topk_state),
+                                  reinterpret_cast<int2*>(ws + lay.topk_counts), topk_max_chunks(d)};
+        return launch_topk(d, a.ut, a.sc_begin, a.sc_end, a.scores, sel, sel_count, st, nullptr, &scratch);
+    }
+    const int tiles_u = (max_units + a.U - 1) / a.U;
+    const dim3 grid(static_cast<unsigned>(a.n_ranges), static_cast<unsigned>(tiles_u));
     switch (d.g) {
     case 1: e = run_tok_passes<1>(grid, rows, tf, tk, a, st); break;
     case 2: e = run_tok_passes<2>(grid, rows, tf, tk, a, st); break;
