@@ -75,8 +75,8 @@ WsLayout ws_layout(const Derived& d)
     w.tok_pack_k = take(pack);
     w.tok_pack_v = take(pack);
     w.tok_count = take(tok ? static_cast<size_t>(d.M) * sizeof(int32_t) : 0);
-    w.topk_hist = take(tok ? static_cast<size_t>(d.M) * 256 * sizeof(int32_t) : 0);
-    w.topk_state = take(tok ? static_cast<size_t>(d.M) * 4 * sizeof(int32_t) : 0);
+    w.topk_hist = take(tok ? static_cast<size_t>(d.M) * kTopkPasses * 256 * sizeof(int32_t) : 0);
+    w.topk_state = take(tok ? static_cast<size_t>(d.M) * (kTopkPasses + 1) * 4 * sizeof(int32_t) : 0);
     w.topk_counts = take(tok ? static_cast<size_t>(d.M) * topk_max_chunks(d) * 2 * sizeof(int32_t) : 0);
     w.stats = take(static_cast<size_t>(d.M) * d.Hq * 2 * sizeof(float));
     w.scores = take(static_cast<size_t>(d.M) * d.nb * sizeof(float));

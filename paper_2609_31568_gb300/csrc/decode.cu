@@ -704,7 +704,7 @@ size_t decode_ws_bytes(const Derived& d, int splits)
     off = align_up(off + cap * sizeof(float), kAlign);                          // scores
     off = align_up(off + static_cast<size_t>(d.Hq) * splits * 130 * sizeof(float), kAlign);
     off = align_up(off + static_cast<size_t>(d.Hq) * ((cap + kDecStat - 1) / kDecStat) * sizeof(float2), kAlign);  // zpart
-    off = align_up(off + (256 + 4) * sizeof(int32_t), kAlign);                                    // top-k hist, state
+    off = align_up(off + (kTopkPasses * 256 + (kTopkPasses + 1) * 4) * sizeof(int32_t), kAlign);  // top-k hist, state
     off = align_up(off + static_cast<size_t>(topk_max_chunks(d)) * sizeof(int2), kAlign);          // top-k counts
     return off;
 }
@@ -749,7 +749,7 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
     a.part = reinterpret_cast<float*>(ws + take(static_cast<size_t>(d.Hq) * kDecSplits * 130 * sizeof(float)));
     a.zpart = reinterpret_cast<float2*>(
         ws + take(static_cast<size_t>(d.Hq) * ((cap + kDecStat - 1) / kDecStat) * sizeof(float2)));
-    int32_t* tk_hist = reinterpret_cast<int32_t*>(ws + take((256 + 4) * sizeof(int32_t)));
+    int32_t* tk_hist = reinterpret_cast<int32_t*>(ws + take((kTopkPasses * 256 + (kTopkPasses + 1) * 4) * sizeof(int32_t)));
     int2* tk_counts = reinterpret_cast<int2*>(ws + take(static_cast<size_t>(topk_max_chunks(d)) * sizeof(int2)));
 
     const auto* qb = static_cast<const __nv_bfloat16*>(q);
@@ -800,7 +800,7 @@ cudaError_t launch_decode_step(const Derived& d, int64_t t, const void* q, const
         du.B = 1;
         du.nb = d.N;
         const Units ut{a.units, a.units + 2, 0, d.N, 1, static_cast<int>(d.N)};
-        const TopkScratch scratch{tk_hist, tk_hist + 256, tk_counts, topk_max_chunks(du)};
+        const TopkScratch scratch{tk_hist, tk_hist + kTopkPasses * 256, tk_counts, topk_max_chunks(du)};
         cudaError_t e = launch_topk(du, ut, static_cast<int>(t), static_cast<int>(t + 1), a.scores, a.sel,
                                     a.sel_count, st, a.state + 2, &scratch);
         if (e != cudaSuccess) return e;

@@ -49,8 +49,8 @@ struct WsLayout {
     size_t tok_pack_k;  // bf16 [M][H_kv][slots][128] distant keys of each unit, packed (block size 1 only)
     size_t tok_pack_v;  // bf16 [M][H_kv][slots][128] distant values, packed
     size_t tok_count;   // int32 [M]                  distant keys of each unit
-    size_t topk_hist;   // int32 [M][256]             multi-CTA top-k scratch (block size 1 only)
-    size_t topk_state;  // int32 [M][4]
+    size_t topk_hist;   // int32 [M][kTopkPasses][256] multi-CTA top-k scratch (block size 1 only)
+    size_t topk_state;  // int32 [M][kTopkPasses + 1][4]
     size_t topk_counts; // int2 [M][topk chunks]
     size_t stats;       // fp32 [M][H_q][2]  (row max, 1 / row sum)
     size_t scores;      // fp32 [M][nb]
@@ -172,9 +172,11 @@ cudaError_t launch_sparse_prefill(const Derived& d, int mode, int64_t tok_begin,
                                   uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 cudaError_t launch_wait_selftest(uint8_t* ws, uint64_t timeout_ns, cudaStream_t st);
 // Scratch of the multi-CTA top-k (units with more than 64K candidates).
+// Radix passes of the multi-CTA top-k (8-bit digits of a 32-bit key).
+constexpr int kTopkPasses = 4;
 struct TopkScratch {
-    int32_t* hist;    // [units][256]
-    int32_t* state;   // [units][4]
+    int32_t* hist;    // [units][kTopkPasses][256]
+    int32_t* state;   // [units][kTopkPasses + 1][4]
     int2* counts;     // [units][max_chunks]
     int max_chunks;   // topk_max_chunks(d)
 };

@@ -552,6 +552,7 @@ struct TopkState {
     int done;         // 1: the unit's output is already complete
     int pad;
 };
+static_assert(sizeof(TopkState) == 4 * sizeof(int32_t), "TopkState is four int32 words");
 
 __device__ __forceinline__ bool unit_cands(const SelArgs& a, int ui, int* u, int64_t* lo, int64_t* hi)
 {
@@ -567,7 +568,10 @@ __device__ __forceinline__ bool unit_cands(const SelArgs& a, int ui, int* u, int
 }
 
 // Per unit: small candidate sets are written out directly; otherwise the
-// radix state starts (prefix 0, need k) and the histogram is cleared.
+// radix state starts (prefix 0, need k) and the four passes' histograms are
+// cleared. state[u][i] is the state after the digits of i passes are fixed;
+// the kernel that first needs state i + 1 derives it from state i and the
+// histogram of pass i (its CTA 0 stores it for the kernels after it).
 __global__ void __launch_bounds__(256) k_topk_init(SelArgs a, int32_t* __restrict__ sel,
                                                     int32_t* __restrict__ sel_count, int32_t* __restrict__ hist,
                                                     TopkState* __restrict__ state)
@@ -577,34 +581,65 @@ __global__ void __launch_bounds__(256) k_topk_init(SelArgs a, int32_t* __restric
     int64_t lo, hi;
     if (!unit_cands(a, blockIdx.x, &u, &lo, &hi)) return;
     const int64_t n = hi - lo;
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[u * 256 + i] = 0;
+    for (int i = threadIdx.x; i < kTopkPasses * 256; i += blockDim.x) hist[u * kTopkPasses * 256 + i] = 0;
     if (n <= a.k) {
         int32_t* out = sel + static_cast<int64_t>(u) * a.k;
         for (int i = threadIdx.x; i < a.k; i += blockDim.x) out[i] = (i < n) ? static_cast<int32_t>(lo + i) : -1;
         if (threadIdx.x == 0) {
             sel_count[u] = static_cast<int32_t>(n);
-            state[u] = TopkState{0u, 0, 1, 0};
+            state[u * (kTopkPasses + 1)] = TopkState{0u, 0, 1, 0};
         }
     } else if (threadIdx.x == 0) {
-        state[u] = TopkState{0u, a.k, 0, 0};
+        state[u * (kTopkPasses + 1)] = TopkState{0u, a.k, 0, 0};
     }
 }
 
-// One radix pass: per-warp histograms of the digit at `shift` of the keys that
-// match the prefix, added into the unit's histogram.
+// State after pass p (p >= 1): the digit of the k-th largest key at the
+// shift of pass p - 1, from that pass's histogram and the state before it
+// (the largest digit d whose keys, with those above it, reach `need`).
+// Every thread of the CTA returns it; CTA 0 stores it.
+__device__ TopkState topk_state_after(const int32_t* __restrict__ hist_u, TopkState* __restrict__ state_u,
+                                      int p, bool store)
+{
+    __shared__ int h[256];
+    __shared__ TopkState s_st;
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) h[i] = hist_u[(p - 1) * 256 + i];
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        TopkState stt = state_u[p - 1];
+        int need = stt.need, cum = 0, d = 255;
+        for (; d > 0; --d) {
+            if (cum + h[d] >= need) break;
+            cum += h[d];
+        }
+        stt.need = need - cum;
+        stt.prefix |= static_cast<uint32_t>(d) << (24 - 8 * (p - 1));
+        s_st = stt;
+        if (store) state_u[p] = stt;
+    }
+    __syncthreads();
+    return s_st;
+}
+
+// Radix pass p (shift 24 - 8 p): per-warp histograms of the digit at `shift`
+// of the keys that match the prefix fixed by the passes before, added into
+// the unit's histogram of pass p.
 __global__ void __launch_bounds__(kChunkThreads) k_topk_hist(SelArgs a, const float* __restrict__ scores,
                                                              int32_t* __restrict__ hist,
-                                                             const TopkState* __restrict__ state, int shift)
+                                                             TopkState* __restrict__ state, int p)
 {
     __shared__ int wh[kChunkThreads / 32][256];
     if (a.gate && !*a.gate) return;
     int u;
     int64_t lo, hi;
     if (!unit_cands(a, blockIdx.y, &u, &lo, &hi)) return;
-    const TopkState stt = state[u];
-    if (stt.done) return;
+    TopkState* su = state + u * (kTopkPasses + 1);
+    int32_t* hu = hist + u * kTopkPasses * 256;
+    if (su[0].done) return;
     const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * kChunk;
     if (c0 >= hi) return;
+    const int shift = 24 - 8 * p;
+    const TopkState stt = p == 0 ? su[0] : topk_state_after(hu, su, p, blockIdx.x == 0);
     const int64_t c1 = (c0 + kChunk < hi) ? c0 + kChunk : hi;
     const int warp = threadIdx.x >> 5;
     for (int i = threadIdx.x; i < (kChunkThreads / 32) * 256; i += blockDim.x) (&wh[0][0])[i] = 0;
@@ -627,49 +662,26 @@ __global__ void __launch_bounds__(kChunkThreads) k_topk_hist(SelArgs a, const fl
     for (int i = threadIdx.x; i < 256; i += blockDim.x) {
         int c = 0;
         for (int w = 0; w < kChunkThreads / 32; ++w) c += wh[w][i];
-        if (c) atomicAdd(&hist[u * 256 + i], c);
-    }
-}
-
-// The digit of the k-th largest key, from the unit's histogram; clears it.
-__global__ void __launch_bounds__(256) k_topk_pick(SelArgs a, int32_t* __restrict__ hist,
-                                                    TopkState* __restrict__ state, int shift)
-{
-    if (a.gate && !*a.gate) return;
-    int u;
-    int64_t lo, hi;
-    if (!unit_cands(a, blockIdx.x, &u, &lo, &hi)) return;
-    if (state[u].done) return;
-    __shared__ int h[256];
-    h[threadIdx.x] = hist[u * 256 + threadIdx.x];
-    hist[u * 256 + threadIdx.x] = 0;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        TopkState stt = state[u];
-        int need = stt.need, cum = 0, d = 255;
-        for (; d > 0; --d) {
-            if (cum + h[d] >= need) break;
-            cum += h[d];
-        }
-        stt.need = need - cum;
-        stt.prefix |= static_cast<uint32_t>(d) << shift;
-        state[u] = stt;
+        if (c) atomicAdd(&hu[p * 256 + i], c);
     }
 }
 
 // Counts per chunk of the keys above the k-th key T and of the keys equal to it.
+// The k-th key T is the prefix after the last pass (derived here, stored by CTA 0).
 __global__ void __launch_bounds__(kChunkThreads) k_topk_count(SelArgs a, const float* __restrict__ scores,
-                                                              const TopkState* __restrict__ state,
+                                                              const int32_t* __restrict__ hist,
+                                                              TopkState* __restrict__ state,
                                                               int2* __restrict__ counts, int max_chunks)
 {
     if (a.gate && !*a.gate) return;
     int u;
     int64_t lo, hi;
     if (!unit_cands(a, blockIdx.y, &u, &lo, &hi)) return;
-    const TopkState stt = state[u];
-    if (stt.done) return;
+    TopkState* su = state + u * (kTopkPasses + 1);
+    if (su[0].done) return;
     const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * kChunk;
     if (c0 >= hi) return;
+    const TopkState stt = topk_state_after(hist + u * kTopkPasses * 256, su, kTopkPasses, blockIdx.x == 0);
     const int64_t c1 = (c0 + kChunk < hi) ? c0 + kChunk : hi;
     const float* sc = scores + static_cast<int64_t>(u) * a.nb;
     int gt = 0, eq = 0;
@@ -708,8 +720,8 @@ __global__ void __launch_bounds__(32) k_topk_scan(SelArgs a, const TopkState* __
     int u;
     int64_t lo, hi;
     if (!unit_cands(a, blockIdx.x, &u, &lo, &hi)) return;
-    const TopkState stt = state[u];
-    if (stt.done) return;
+    if (state[u * (kTopkPasses + 1)].done) return;
+    const TopkState stt = state[u * (kTopkPasses + 1) + kTopkPasses];
     const int n_chunks = static_cast<int>((hi - lo + kChunk - 1) / kChunk);
     int2* cu = counts + static_cast<int64_t>(u) * max_chunks;
     __shared__ int s_total;
@@ -743,8 +755,8 @@ __global__ void __launch_bounds__(kChunkThreads) k_topk_emit(SelArgs a, const fl
     int u;
     int64_t lo, hi;
     if (!unit_cands(a, blockIdx.y, &u, &lo, &hi)) return;
-    const TopkState stt = state[u];
-    if (stt.done) return;
+    if (state[u * (kTopkPasses + 1)].done) return;
+    const TopkState stt = state[u * (kTopkPasses + 1) + kTopkPasses];
     const int64_t c0 = lo + static_cast<int64_t>(blockIdx.x) * kChunk;
     if (c0 >= hi) return;
     const int64_t c1 = (c0 + kChunk < hi) ? c0 + kChunk : hi;
@@ -901,11 +913,9 @@ cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_
     const int mc = scratch->max_chunks;
     const dim3 grid(static_cast<unsigned>(mc), static_cast<unsigned>(max_units));
     k_topk_init<<<max_units, 256, 0, st>>>(a, sel, sel_count, scratch->hist, state);
-    for (int shift = 24; shift >= 0; shift -= 8) {
-        k_topk_hist<<<grid, kChunkThreads, 0, st>>>(a, scores, scratch->hist, state, shift);
-        k_topk_pick<<<max_units, 256, 0, st>>>(a, scratch->hist, state, shift);
-    }
-    k_topk_count<<<grid, kChunkThreads, 0, st>>>(a, scores, state, scratch->counts, mc);
+    for (int p = 0; p < kTopkPasses; ++p)
+        k_topk_hist<<<grid, kChunkThreads, 0, st>>>(a, scores, scratch->hist, state, p);
+    k_topk_count<<<grid, kChunkThreads, 0, st>>>(a, scores, scratch->hist, state, scratch->counts, mc);
     k_topk_scan<<<max_units, 32, 0, st>>>(a, state, scratch->counts, mc, sel, sel_count);
     k_topk_emit<<<grid, kChunkThreads, 0, st>>>(a, scores, state, scratch->counts, mc, sel);
     return cudaGetLastError();
