@@ -209,20 +209,29 @@ def test_qwen2_7b_head_shape_end_to_end(mode):
     assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
 
 
+# bf16 spike key values 14.0, 22.0 and 32.0: against a query coordinate of 8
+# the spike's logit lies about 12, 20 and 30 log2 units above the rows' other
+# logits. The first stays on the softmax's fast path (every p of the tile at
+# most 2^16, the running max kept), the others fail its sum test and take the
+# exact path (raise, O rescale).
+SPIKES = (0x4160, 0x41B0, 0x4200)
+
+
+@pytest.mark.parametrize("spike", SPIKES)
 @pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
-def test_attention_max_jump_in_alternate_rows(mode):
+def test_attention_max_jump_in_alternate_rows(mode, spike):
     """Rows whose running max jumps in a later key tile next to rows whose max
     does not: even rows get a large score against a few spike keys (the online
-    softmax of Sec. V-A3 must raise their max and rescale their partial sums),
-    odd rows score exactly 0 against them. Both kinds of row share each group
-    of 32 consecutive rows."""
+    softmax of Sec. V-A3 must raise their max and rescale their partial sums,
+    or keep a lower max with large terms), odd rows score exactly 0 against
+    them. Both kinds of row share each group of 32 consecutive rows."""
     w, q, k, v, _ = inputs("gqa4-4k")
     q = q.copy()
     k = k.copy()
     spikes = np.arange(200, w.n_tokens, 512)
     k[spikes] = 0
-    k[spikes, :, 0] = 0x4200  # bf16 32.0
-    q[0::2, :, 0] = 0x4100    # bf16 8.0: score 256 against a spike key
+    k[spikes, :, 0] = spike
+    q[0::2, :, 0] = 0x4100    # bf16 8.0: score 8 x spike against a spike key
     q[1::2, :, 0] = 0         # score 0 against a spike key
     dev = [torch.from_numpy(x).view(torch.bfloat16).cuda() for x in (q, k, v)]
     rows = np.arange(w.n_tokens)
@@ -231,7 +240,7 @@ def test_attention_max_jump_in_alternate_rows(mode):
     out = _prefill_on(w, mode, dev, us, len(us) - 1, ref["sel"], ref["sel_count"])
     got = to_f64_bf16(out)
     mx, mean = attn_errors(got, ref["attn"])
-    print(f"mode={mode}: max {mx:.3e} mean {mean:.3e}")
+    print(f"mode={mode} spike={spike:#x}: max {mx:.3e} mean {mean:.3e}")
     assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
 
 
