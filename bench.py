@@ -89,9 +89,9 @@ def launches(w, selects: int = 1, builds: int = 1) -> dict:
     list)."""
     tok = w.block_size == 1
     build = (2 if tok else 3) + (1 if w.max_cluster_subchunks > 1 else 0)
-    # the top-k is one kernel, or 12 (init, 4 x (histogram, pick), count, scan,
+    # the top-k is one kernel, or 8 (init, 4 histogram passes, count, scan,
     # emit) for units of more than 64K candidates
-    topk = 12 if tok and w.n_blocks > 65536 else 1
+    topk = 8 if tok and w.n_blocks > 65536 else 1
     select = (4 if tok else 3) + topk
     attend = 3 if tok else 1
     return {"build_reps": build * builds, "select": select * selects, "attend": attend * selects,
