@@ -19,6 +19,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -136,19 +137,29 @@ def key_counts(w, unit_start, n_units, sel, cnt, per_subchunk):
     return total
 
 
+def kernel_source_hash(path: str) -> str:
+    """sha256[:16] of a CUDA source with its comments and blank lines removed:
+    a change to the code changes it, a change to a comment does not."""
+    with open(path) as f:
+        txt = f.read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    txt = re.sub(r"//[^\n]*", "", txt)
+    code = "\n".join(ln.rstrip() for ln in txt.splitlines() if ln.strip())
+    return hashlib.sha256(code.encode()).hexdigest()[:16]
+
+
 def profile_counters(workload_name: str) -> dict:
     """ncu counters of the attention kernel on this workload, from the
     machine-readable sidecar committed beside its summary
     (profiles/attn_<workload>_ncu.json). Empty when there is none or when the
-    kernel source changed since the capture (its hash is stored with it)."""
+    kernel's code changed since the capture (the hash of its source without
+    comments is stored with it)."""
     path = os.path.join(PROFILE_DIR, f"attn_{workload_name}_ncu.json")
     if not os.path.exists(path):
         return {}
-    with open(KERNEL_SRC, "rb") as f:
-        sha = hashlib.sha256(f.read()).hexdigest()[:16]
     with open(path) as f:
         rec = json.load(f)
-    return rec if rec.get("kernel_source_sha16") == sha else {}
+    return rec if rec.get("kernel_code_sha16") == kernel_source_hash(KERNEL_SRC) else {}
 
 
 class ClockSampler:

@@ -52,8 +52,10 @@ constexpr uint32_t kSegBytes = 64 * 128;      // one 64-row x 64-column box
 constexpr float kRescaleThreshold = 8.0f;     // log2 units
 constexpr float kFastSumLimit = 65536.0f;     // 2^16: largest tile sum kept on the fast path
 // Softmax exponentials of column pair i go to the FMA pipe (exp2_poly2) when
-// bit (i % 8) is set, else to the special-function unit; the split balances
-// the two units, which otherwise bound the softmax.
+// bit (i % 8) is set, else to the special-function unit. On sm_103 the
+// special-function unit is not what bounds the softmax (moving any share of
+// the exponentials only added issue slots in measurements), so none are moved
+// by default.
 #ifndef SCALE_SOFT_EXP_MASK
 #define SCALE_SOFT_EXP_MASK 0x00
 #endif

@@ -4,7 +4,6 @@ kernel source is unchanged, the launch counts follow the path's kernels, the
 Algorithm 2 loop issues one selection and attention call per unit, and the
 selection agreement counts near-ties apart from mismatches."""
 
-import hashlib
 import json
 import os
 import sys
@@ -18,17 +17,19 @@ import bench  # noqa: E402
 from synth import workload  # noqa: E402
 
 
-def test_profile_counters_follow_the_kernel_source(tmp_path, monkeypatch):
+def test_profile_counters_follow_the_kernel_code(tmp_path, monkeypatch):
     src = tmp_path / "attn.cu"
-    src.write_bytes(b"// kernel v1\n")
-    sha = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    src.write_text("// kernel\nint v = 1;  // one\n")
     (tmp_path / "attn_wl-a_ncu.json").write_text(json.dumps(
-        {"kernel_source_sha16": sha, "traffic_bytes_per_launch": 12345, "tensor_pipe_active_pct": 70.0}))
+        {"kernel_code_sha16": bench.kernel_source_hash(str(src)), "traffic_bytes_per_launch": 12345,
+         "tensor_pipe_active_pct": 70.0}))
     monkeypatch.setattr(bench, "KERNEL_SRC", str(src))
     monkeypatch.setattr(bench, "PROFILE_DIR", str(tmp_path))
     assert bench.profile_counters("wl-a")["traffic_bytes_per_launch"] == 12345
     assert bench.profile_counters("wl-b") == {}  # no capture of that workload
-    src.write_bytes(b"// kernel v2\n")  # changed since the capture
+    src.write_text("/* the kernel */\n\nint v = 1;  // first\n")  # comments only: same code
+    assert bench.profile_counters("wl-a")["tensor_pipe_active_pct"] == 70.0
+    src.write_text("// kernel\nint v = 2;  // one\n")  # the code changed since the capture
     assert bench.profile_counters("wl-a") == {}
 
 
@@ -38,7 +39,7 @@ def test_committed_sidecars_are_valid_json():
         if name.endswith(".json"):
             with open(os.path.join(d, name)) as f:
                 rec = json.load(f)
-            assert len(rec["kernel_source_sha16"]) == 16
+            assert len(rec["kernel_code_sha16"]) == 16
 
 
 def test_algorithm2_loop_calls():
