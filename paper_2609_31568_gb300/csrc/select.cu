@@ -543,7 +543,8 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
 // ---- top-k over many candidates per unit: the same radix select and ordered
 // output as k_topk, spread over CTAs of kChunk candidates (grid y = unit).
 
-constexpr int kChunk = 8192;
+constexpr int kChunk = 2048;              // candidates per CTA and pass
+constexpr int64_t kMultiCtaMin = 65536;   // more candidates than this: the multi-CTA form
 constexpr int kChunkThreads = 256;
 
 struct TopkState {
@@ -724,23 +725,35 @@ __global__ void __launch_bounds__(32) k_topk_scan(SelArgs a, const TopkState* __
     const TopkState stt = state[u * (kTopkPasses + 1) + kTopkPasses];
     const int n_chunks = static_cast<int>((hi - lo + kChunk - 1) / kChunk);
     int2* cu = counts + static_cast<int64_t>(u) * max_chunks;
-    __shared__ int s_total;
-    if (threadIdx.x == 0) {
-        int eq_before = 0, pos = 0;
-        for (int c = 0; c < n_chunks; ++c) {
-            const int2 ge = cu[c];
-            int take = stt.need - eq_before;
-            take = take < 0 ? 0 : (take > ge.y ? ge.y : take);
-            eq_before += ge.y;
-            cu[c] = make_int2(pos, take);
-            pos += ge.x + take;
+    // Two prefix sums over the chunks, 32 at a time with the totals carried:
+    // the equal keys before each chunk (how many of its equal keys it takes
+    // follows), then the picks before it (its output position).
+    const int lane = threadIdx.x;
+    int eq_run = 0, pos_run = 0;
+    for (int c0 = 0; c0 < n_chunks; c0 += 32) {
+        const int c = c0 + lane;
+        const int2 ge = c < n_chunks ? cu[c] : make_int2(0, 0);
+        int eq_inc = ge.y;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, eq_inc, o);
+            if (lane >= o) eq_inc += y;
         }
-        s_total = pos;
-        sel_count[u] = pos;
+        const int eq_before = eq_run + eq_inc - ge.y;
+        int take = stt.need - eq_before;
+        take = take < 0 ? 0 : (take > ge.y ? ge.y : take);
+        const int picks = ge.x + take;
+        int pos_inc = picks;
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xFFFFFFFFu, pos_inc, o);
+            if (lane >= o) pos_inc += y;
+        }
+        if (c < n_chunks) cu[c] = make_int2(pos_run + pos_inc - picks, take);
+        eq_run += __shfl_sync(0xFFFFFFFFu, eq_inc, 31);
+        pos_run += __shfl_sync(0xFFFFFFFFu, pos_inc, 31);
     }
-    __syncwarp();
+    if (lane == 0) sel_count[u] = pos_run;
     int32_t* out = sel + static_cast<int64_t>(u) * a.k;
-    for (int i = s_total + threadIdx.x; i < a.k; i += 32) out[i] = -1;
+    for (int i = pos_run + lane; i < a.k; i += 32) out[i] = -1;
 }
 
 // Ordered output of one chunk: every warp owns a contiguous segment (lane l
@@ -904,7 +917,7 @@ cudaError_t launch_topk(const Derived& d, const Units& ut, int sc_begin, int sc_
     a.sigma = d.sigma;
     const int max_units = sc_end - sc_begin;
     if (max_units <= 0) return cudaSuccess;
-    if (!scratch || d.nb <= 8 * kChunk) {
+    if (!scratch || d.nb <= kMultiCtaMin) {
         k_topk<<<max_units, kTopkThreads, 0, st>>>(a, scores, sel, sel_count);
         return cudaGetLastError();
     }

@@ -61,6 +61,7 @@ struct TokArgs {
     int range;          // tokens per CTA (128 g, at most 1024)
     int n_ranges;
     int N, n_sink, n_local;
+    int head_split;     // k_tok_score_s pass 0: one KV head per CTA (grid z)
     float scale2;       // sigma * log2(e)
     float2* part;       // [M][H_q][n_ranges] (max, sum) in log2 units
     const float2* stats;  // [M][H_q] (max, 1 / sum)
@@ -356,7 +357,14 @@ k_tok_score(const __grid_constant__ CUtensorMap tf, const __grid_constant__ CUte
 // 96 KB. Pass 0 keeps a running (max, sum) per column in each token's thread
 // and merges the 128 threads once per KV head (a fixed shuffle tree, then
 // the four warps in order); pass 1 keeps each token's votes in registers.
-constexpr int kNc = 16;                        // (unit, head) columns of a small tile
+// For parallelism when the sequence has few token ranges, pass 0 then runs
+// one CTA per KV head (grid z; its partials are per (unit, head) anyway) and
+// pass 1 (NARROW) one CTA per 128 tokens (the votes are per token); with many
+// ranges the CTAs keep all KV heads and whole ranges, which amortises the
+// fingerprint loads and the pipeline start over more key tiles.
+constexpr int kNc = 16;
+constexpr int kRange1 = 128;                   // narrow pass 1: tokens per CTA
+constexpr int kFewRanges = 1024;               // below this many ranges: the split grids                        // (unit, head) columns of a small tile
 constexpr uint32_t kFsHalf = 3 * kNc * 128;    // one 64-column half of the 48-row operand: 6 KB
 constexpr uint32_t kOffFs = 0;                 // fingerprint parts, 12 KB
 constexpr uint32_t kOffKs = 2 * kFsHalf;       // 2 key stages (a multiple of 1024)
@@ -372,7 +380,7 @@ __device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2
     m = mn;
 }
 
-template <int PASS, int G>
+template <int PASS, int G, bool NARROW>
 __global__ void __launch_bounds__(kTokThreads, 2)
 k_tok_score_s(const __grid_constant__ CUtensorMap tfs, const __grid_constant__ CUtensorMap tk, const TokArgs a)
 {
@@ -391,8 +399,12 @@ k_tok_score_s(const __grid_constant__ CUtensorMap tfs, const __grid_constant__ C
     if (u0 >= u_end) return;
     const int n_u = (u_end - u0 < US) ? u_end - u0 : US;
     const int x = blockIdx.x;
-    const int r0 = x * a.range;
-    const int r1 = (r0 + a.range < a.N) ? r0 + a.range : a.N;
+    const int rlen = (PASS == 1 && NARROW) ? kRange1 : a.range;
+    const int r0 = x * rlen;
+    const int r1 = (r0 + rlen < a.N) ? r0 + rlen : a.N;
+    const bool split = PASS == 0 && a.head_split;  // KV heads of this CTA
+    const int j_lo = split ? static_cast<int>(blockIdx.z) : 0;
+    const int j_hi = split ? j_lo + 1 : a.Hkv;
     const int64_t w_max = window_start(a, u0 + n_u - 1);
     const int c_hi = static_cast<int>(w_max < r1 ? w_max : r1);
     const bool work = c_hi > r0 && c_hi > a.n_sink;
@@ -439,8 +451,8 @@ k_tok_score_s(const __grid_constant__ CUtensorMap tfs, const __grid_constant__ C
             tma_prefetch_desc(&tk);
             int gt = 0;
             int issued_k0 = 0, issued_k1 = 0, issued_f = 0;
-            for (int j = 0; j < a.Hkv && !abort_flag; ++j) {
-                if (j > 0 && !mbar_wait_bounded(&bars.f_empty, (j - 1) & 1, a.timeout_ns, &abort_flag)) {
+            for (int j = j_lo; j < j_hi && !abort_flag; ++j) {
+                if (j > j_lo && !mbar_wait_bounded(&bars.f_empty, (j - j_lo - 1) & 1, a.timeout_ns, &abort_flag)) {
                     tok_fail(&abort_flag, a.status);
                     break;
                 }
@@ -482,8 +494,8 @@ k_tok_score_s(const __grid_constant__ CUtensorMap tfs, const __grid_constant__ C
             constexpr uint64_t kStep = kTile >> 4;
             bool ok = true;
             int gt = 0;
-            for (int j = 0; ok && j < a.Hkv; ++j) {
-                if (!mbar_wait_bounded(&bars.f_full, j & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
+            for (int j = j_lo; ok && j < j_hi; ++j) {
+                if (!mbar_wait_bounded(&bars.f_full, (j - j_lo) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
                 for (int i = 0; i < n_tiles; ++i, ++gt) {
                     const int st = gt & 1;
                     if (!mbar_wait_bounded(&bars.k_full[st], (gt >> 1) & 1, a.timeout_ns, &abort_flag)) { ok = false; break; }
@@ -521,7 +533,7 @@ k_tok_score_s(const __grid_constant__ CUtensorMap tfs, const __grid_constant__ C
                 z[c] = (__uint_as_float(p0[c]) + __uint_as_float(p1[c])) + __uint_as_float(p2[c]);
         };
         if (PASS == 0) {
-            for (int j = 0; j < a.Hkv; ++j) {
+            for (int j = j_lo; j < j_hi; ++j) {
                 float m[kNc], sm[kNc];
 #pragma unroll
                 for (int c = 0; c < kNc; ++c) {
@@ -582,7 +594,7 @@ k_tok_score_s(const __grid_constant__ CUtensorMap tfs, const __grid_constant__ C
             }
         } else {
             // votes of this thread's token in each key tile of the range, per unit
-            constexpr int kTiles = G <= 8 ? G : 8;  // a.range / 128
+            constexpr int kTiles = NARROW ? kRange1 / 128 : (G < 8 ? G : 8);  // the range's key tiles
             float vote[kTiles][US];
 #pragma unroll
             for (int i = 0; i < kTiles; ++i)
@@ -728,20 +740,36 @@ cudaError_t run_tok_passes(dim3 grid, int64_t rows, const CUtensorMap& tf, const
 // kSmallUnits units.
 constexpr int kSmallUnits = 16;
 
-template <int G>
-cudaError_t run_tok_passes_s(dim3 grid, int64_t rows, const CUtensorMap& tfs, const CUtensorMap& tk,
-                             const TokArgs& a, cudaStream_t st)
+template <int G, bool NARROW>
+cudaError_t run_tok_passes_s(dim3 grid0, dim3 grid1, int64_t rows, const CUtensorMap& tfs,
+                             const CUtensorMap& tk, const TokArgs& a, cudaStream_t st)
 {
-    cudaError_t e = cudaFuncSetAttribute(k_tok_score_s<0, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(kSmemTokS));
+    cudaError_t e = cudaFuncSetAttribute(k_tok_score_s<0, G, NARROW>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmemTokS));
     if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_tok_score_s<1, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(k_tok_score_s<1, G, NARROW>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(kSmemTokS));
     if (e != cudaSuccess) return e;
-    k_tok_score_s<0, G><<<grid, kTokThreads, kSmemTokS, st>>>(tfs, tk, a);
+    k_tok_score_s<0, G, NARROW><<<grid0, kTokThreads, kSmemTokS, st>>>(tfs, tk, a);
     k_tok_merge<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a);
-    k_tok_score_s<1, G><<<grid, kTokThreads, kSmemTokS, st>>>(tfs, tk, a);
+    k_tok_score_s<1, G, NARROW><<<grid1, kTokThreads, kSmemTokS, st>>>(tfs, tk, a);
     return cudaGetLastError();
+}
+
+template <int G>
+cudaError_t run_tok_passes_s(const Derived& d, int tiles, int64_t rows, const CUtensorMap& tfs,
+                             const CUtensorMap& tk, TokArgs a, cudaStream_t st)
+{
+    const unsigned nt = static_cast<unsigned>(tiles);
+    if (a.n_ranges < kFewRanges) {
+        a.head_split = 1;
+        return run_tok_passes_s<G, true>(dim3(static_cast<unsigned>(a.n_ranges), nt, static_cast<unsigned>(d.Hkv)),
+                                         dim3(static_cast<unsigned>((d.N + kRange1 - 1) / kRange1), nt, 1), rows,
+                                         tfs, tk, a, st);
+    }
+    a.head_split = 0;
+    const dim3 g(static_cast<unsigned>(a.n_ranges), nt, 1);
+    return run_tok_passes_s<G, false>(g, g, rows, tfs, tk, a, st);
 }
 
 }  // namespace
@@ -772,6 +800,7 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
     a.N = static_cast<int>(d.N);
     a.n_sink = d.n_sink;
     a.n_local = d.n_local;
+    a.head_split = 0;
     a.scale2 = d.sigma * 1.4426950408889634f;
     a.part = reinterpret_cast<float2*>(ws + lay.tok_part);
     a.stats = reinterpret_cast<const float2*>(ws + lay.stats);
@@ -798,17 +827,16 @@ cudaError_t launch_select_tokens(const Derived& d, int mode, int64_t tok_begin, 
         CUtensorMap tfs;
         const uint32_t fbox_s[4] = {64, kNc, 1, 1};
         if (!scale_host::make_dense_bf16_map(&tfs, parts, 4, fdims, fbox_s)) return cudaErrorInvalidValue;
-        const int us = kNc / d.g;
-        const dim3 grid_s(static_cast<unsigned>(a.n_ranges), static_cast<unsigned>((max_units + us - 1) / us));
+        const int tiles = (max_units + kNc / d.g - 1) / (kNc / d.g);
         switch (d.g) {
-        case 1: e = run_tok_passes_s<1>(grid_s, rows, tfs, tk, a, st); break;
-        case 2: e = run_tok_passes_s<2>(grid_s, rows, tfs, tk, a, st); break;
-        case 3: e = run_tok_passes_s<3>(grid_s, rows, tfs, tk, a, st); break;
-        case 4: e = run_tok_passes_s<4>(grid_s, rows, tfs, tk, a, st); break;
-        case 5: e = run_tok_passes_s<5>(grid_s, rows, tfs, tk, a, st); break;
-        case 6: e = run_tok_passes_s<6>(grid_s, rows, tfs, tk, a, st); break;
-        case 7: e = run_tok_passes_s<7>(grid_s, rows, tfs, tk, a, st); break;
-        case 8: e = run_tok_passes_s<8>(grid_s, rows, tfs, tk, a, st); break;
+        case 1: e = run_tok_passes_s<1>(d, tiles, rows, tfs, tk, a, st); break;
+        case 2: e = run_tok_passes_s<2>(d, tiles, rows, tfs, tk, a, st); break;
+        case 3: e = run_tok_passes_s<3>(d, tiles, rows, tfs, tk, a, st); break;
+        case 4: e = run_tok_passes_s<4>(d, tiles, rows, tfs, tk, a, st); break;
+        case 5: e = run_tok_passes_s<5>(d, tiles, rows, tfs, tk, a, st); break;
+        case 6: e = run_tok_passes_s<6>(d, tiles, rows, tfs, tk, a, st); break;
+        case 7: e = run_tok_passes_s<7>(d, tiles, rows, tfs, tk, a, st); break;
+        case 8: e = run_tok_passes_s<8>(d, tiles, rows, tfs, tk, a, st); break;
         default: return cudaErrorInvalidValue;
         }
         if (e == cudaSuccess) e = cudaGetLastError();
