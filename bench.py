@@ -366,7 +366,7 @@ def loop_calls(w, mode_sub: bool):
 # (Algorithm 2 loop in both modes, plus the whole-sequence launches), with the
 # GPU selection compared with the oracle's where steps (a)-(c) fit in seconds.
 OTHER_CONFIGS = (("gqa4-4k", True), ("llama8b-32k", True), ("llama8b-64k-32l", False), ("llama8b-1m", True),
-                 ("llama8b-128k-tok", True))
+                 ("llama8b-128k-tok", True), ("llama8b-1m-tok", False))
 OTHER_STEPS, OTHER_WARMUP = 3, 3
 
 

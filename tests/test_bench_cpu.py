@@ -112,6 +112,7 @@ def test_other_configs_compacts_each_side_run(monkeypatch):
     assert [c[c.index("--workload") + 1] for c in calls] == [n for n, _ in bench.OTHER_CONFIGS]
     assert all("--no-other-configs" in c for c in calls)
     assert ("--selection-check" in calls[2]) is False  # the stack runs no oracle check
+    assert ("--selection-check" in calls[-1]) is False  # nor 1M tokens at token level
     l32 = got["llama8b-32k"]
     assert l32["cluster"]["ttft_ms"] == 6.0 and l32["subchunk"]["ttft_ms"] == 5.0
     assert l32["cluster"]["batched_ms"] == 2.7 and l32["subchunk"]["select_ms"] == 3.0
