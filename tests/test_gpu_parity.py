@@ -296,7 +296,8 @@ TOKEN_CASES = [("gqa4-4k", dict(block_size=1, top_k=64)),
                ("llama8b-32k", dict(block_size=1, top_k=1024)),
                # the paper's model and selection: Qwen2-7B heads (28 on 4 KV heads), token level
                ("gqa4-4k", dict(block_size=1, top_k=128, num_q_heads=28, num_kv_heads=4, n_tokens=2048 + 64)),
-               ("gqa4-4k", dict(block_size=1, top_k=96, num_q_heads=6, num_kv_heads=2, n_tokens=2048 + 64))]
+               ("gqa4-4k", dict(block_size=1, top_k=96, num_q_heads=6, num_kv_heads=2, n_tokens=2048 + 64)),
+               ("gqa4-4k", dict(block_size=1, top_k=64, num_q_heads=16, num_kv_heads=2, n_tokens=2048 + 64))]
 
 
 @pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
@@ -336,6 +337,40 @@ def test_token_attention_parity_on_oracle_selection(name, over, stride, mode):
     mx, mean = attn_errors(got, ref["attn"])
     print(f"{name} {over} mode={mode}: max {mx:.3e} mean {mean:.3e}")
     assert mx <= ATTN_MAX_ABS and mean <= ATTN_MEAN_ABS
+
+
+@pytest.mark.parametrize("mode", [PER_CLUSTER, PER_SUB])
+def test_token_select_range_calls_long_sequence(mode):
+    """Token-level selection by range calls, one outer chunk per call as the
+    Algorithm 2 loop issues them, on a sequence with 1024 token ranges (128K
+    tokens, one query head per KV head): the few-unit scorer then keeps whole
+    ranges and all KV heads in each CTA, and the later units have more than
+    64K candidates (the multi-CTA top-k). Every unit's scores and selection
+    against the oracle's Eq. 9 and top-k."""
+    w, q, k, v, dev = inputs("llama8b-128k-tok", num_q_heads=8, num_kv_heads=8)
+    p = S.params_for(w)
+    buf = S.allocate(p, mode, want_scores=True)
+    for t0 in range(0, w.n_tokens, w.outer_chunk):
+        t1 = min(w.n_tokens, t0 + w.outer_chunk)
+        S.scale_build_reps_range(p, t0, t1, dev[0], dev[1], buf.reps, buf.fingerprints, buf.unit_start,
+                                 buf.n_units, buf.ws)
+        S.select(p, mode, t0, t1, dev[1], buf)
+    torch.cuda.synchronize()
+    assert S.scale_get_device_status(buf.ws) == S.SCALE_OK
+    ref = oracle.run_path(w, q, k, v, per_subchunk=(mode == PER_SUB))
+    n = unit_count(buf, mode, w)
+    assert n == len(ref["sel_count"])
+    same, near = compare_selection(buf.sel_blocks.cpu().numpy()[:n, : w.top_k], buf.sel_count.cpu().numpy()[:n],
+                                   ref)
+    ref_sc = oracle.select(num_q_heads=w.num_q_heads, n_tokens=w.n_tokens, sub_chunk=w.sub_chunk,
+                           block_size=1, top_k=w.top_k, n_sink=w.n_sink, n_local=w.n_local,
+                           select_scale=1.0, per_subchunk=(mode == PER_SUB), reps=ref["reps"],
+                           v=ref["fingerprints"], unit_start=ref["unit_start"], want_scores=True)["scores"]
+    got_sc = buf.sel_scores.cpu().numpy()[:n].astype(np.float64)
+    cand = ~np.isnan(ref_sc)
+    assert np.array_equal(cand, ~np.isnan(got_sc))
+    np.testing.assert_allclose(got_sc[cand], ref_sc[cand], rtol=2e-5, atol=1e-10)
+    print(f"mode={mode}: {n} units, {near} near-tie units differ")
 
 
 def test_token_attention_ignores_invalid_entries():
