@@ -93,7 +93,11 @@ def launches(w, selects: int = 1, builds: int = 1) -> dict:
     # the top-k is one kernel, or 8 (init, 4 histogram passes, count, scan,
     # emit) for units of more than 64K candidates
     topk = 8 if tok and w.n_blocks > 65536 else 1
-    select = (4 if tok else 3) + topk
+    if tok:
+        select = 4 + topk
+    else:
+        # logits, then statistics + vote + top-k in one kernel up to 4096 blocks
+        select = 2 if w.n_blocks <= 4096 and w.num_q_heads <= 256 else 3 + topk
     attend = 3 if tok else 1
     return {"build_reps": build * builds, "select": select * selects, "attend": attend * selects,
             "total": build * builds + (select + attend) * selects}

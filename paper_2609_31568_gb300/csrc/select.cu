@@ -307,9 +307,61 @@ __device__ __forceinline__ uint32_t float_key(float f)
 }
 
 constexpr int kTopkThreads = 1024;
-constexpr int kTopkUnroll = 16;  // independent loads in flight per thread
+constexpr int kSortMax = 4096;     // candidates up to which the top-k sorts instead
 
-constexpr int kSortMax = 4096;     // candidates up to which k_topk sorts instead
+// The k picks among np (a power of two, at most kSortMax) 64-bit keys
+// (~float_key(score), candidate index) in shared memory, written to out in
+// ascending candidate order (candidate i is block lo + i): a bitonic sort puts
+// the picks first (higher score first, equal scores by lower index), their
+// indices are marked in a bitmap (bm: np / 32 + 1 words) and written in order
+// after one scan. Called by all kTopkThreads threads of the CTA.
+__device__ void topk_sort_emit(uint64_t* sk, uint32_t* bm, int np, int64_t lo, int k, int32_t* out)
+{
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int size = 2; size <= np; size <<= 1)
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            for (int i = threadIdx.x; i < np; i += blockDim.x) {
+                const int l = i ^ stride;
+                if (l > i) {
+                    const uint64_t x = sk[i], y = sk[l];
+                    if ((x > y) == ((i & size) == 0)) {
+                        sk[i] = y;
+                        sk[l] = x;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+    for (int w = threadIdx.x; w < np / 32 + 1; w += blockDim.x) bm[w] = 0u;
+    __syncthreads();
+    for (int r = threadIdx.x; r < k; r += blockDim.x) {
+        const uint32_t i = static_cast<uint32_t>(sk[r]);
+        atomicOr(&bm[i >> 5], 1u << (i & 31));
+    }
+    __syncthreads();
+    // ascending output: word t of the bitmap to thread t, exclusive scan of the counts
+    __shared__ int s_wsum[4];
+    const int nwords = (np + 31) / 32;
+    uint32_t word = threadIdx.x < nwords ? bm[threadIdx.x] : 0u;
+    const int c = __popc(word);
+    int inc = c;
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+        if (lane >= o) inc += y;
+    }
+    if (lane == 31 && warp < 4) s_wsum[warp] = inc;
+    __syncthreads();
+    if (threadIdx.x < nwords) {
+        int p = inc - c;
+        for (int w = 0; w < warp; ++w) p += s_wsum[w];
+        while (word) {
+            const int bit = __ffs(word) - 1;
+            word &= word - 1;
+            out[p++] = static_cast<int32_t>(lo + 32 * threadIdx.x + bit);
+        }
+    }
+}
+constexpr int kTopkUnroll = 16;  // independent loads in flight per thread
 
 // One CTA per unit. Up to kSortMax candidates, a bitonic sort in shared
 // memory of the 64-bit keys (~float_key(score), index) puts the picks first
@@ -357,49 +409,7 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
             sk[i] = i < n ? (static_cast<uint64_t>(~float_key(sc[lo + i])) << 32) | static_cast<uint32_t>(i)
                           : ~0ull;  // padding sorts last
         __syncthreads();
-        for (int size = 2; size <= np; size <<= 1)
-            for (int stride = size >> 1; stride > 0; stride >>= 1) {
-                for (int i = threadIdx.x; i < np; i += blockDim.x) {
-                    const int l = i ^ stride;
-                    if (l > i) {
-                        const uint64_t x = sk[i], y = sk[l];
-                        if ((x > y) == ((i & size) == 0)) {
-                            sk[i] = y;
-                            sk[l] = x;
-                        }
-                    }
-                }
-                __syncthreads();
-            }
-        uint32_t* bm = reinterpret_cast<uint32_t*>(hist);  // np / 32 <= 128 words
-        for (int w = threadIdx.x; w < np / 32 + 1; w += blockDim.x) bm[w] = 0u;
-        __syncthreads();
-        for (int r = threadIdx.x; r < a.k; r += blockDim.x) {
-            const uint32_t i = static_cast<uint32_t>(sk[r]);
-            atomicOr(&bm[i >> 5], 1u << (i & 31));
-        }
-        __syncthreads();
-        // ascending output: word t of the bitmap to thread t, exclusive scan of the counts
-        __shared__ int s_wsum[4];
-        const int nwords = (np + 31) / 32;
-        uint32_t word = threadIdx.x < nwords ? bm[threadIdx.x] : 0u;
-        const int c = __popc(word);
-        int inc = c;
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-            if (lane >= o) inc += y;
-        }
-        if (lane == 31 && warp < 4) s_wsum[warp] = inc;
-        __syncthreads();
-        if (threadIdx.x < nwords) {
-            int p = inc - c;
-            for (int w = 0; w < warp; ++w) p += s_wsum[w];
-            while (word) {
-                const int bit = __ffs(word) - 1;
-                word &= word - 1;
-                out[p++] = static_cast<int32_t>(lo + 32 * threadIdx.x + bit);
-            }
-        }
+        topk_sort_emit(sk, reinterpret_cast<uint32_t*>(hist), np, lo, a.k, out);
         if (threadIdx.x == 0) sel_count[u] = a.k;  // n > k: exactly k picks
         return;
     }
@@ -538,6 +548,99 @@ __global__ void __launch_bounds__(kTopkThreads) k_topk(SelArgs a, const float* _
     }
     for (int i = taken + threadIdx.x; i < a.k; i += blockDim.x) out[i] = -1;
     if (threadIdx.x == 0) sel_count[u] = taken;
+}
+
+// Steps (b)-(c) after the logits for units of at most kSortMax candidates,
+// one CTA of kTopkThreads per unit: the per-head max and 1 / sum of k_stats,
+// the soft vote of k_vote (scores written for every block, NaN off the
+// candidates) and the sort path of k_topk, with the same arithmetic in the
+// same order, so scores and selection equal those of the three kernels.
+constexpr int kFusedMaxHeads = 256;
+__global__ void __launch_bounds__(kTopkThreads) k_select_fused(SelArgs a, const float* __restrict__ logits,
+                                                               float* __restrict__ scores,
+                                                               int32_t* __restrict__ sel,
+                                                               int32_t* __restrict__ sel_count)
+{
+    __shared__ float s_m[kFusedMaxHeads], s_inv[kFusedMaxHeads];
+    __shared__ __align__(16) uint64_t sk[kSortMax];
+    __shared__ uint32_t bm[kSortMax / 32 + 1];
+    const int u_first = unit_lower_bound(a.ut, a.sc_begin);
+    const int u_end = unit_lower_bound(a.ut, a.sc_end);
+    const int u = u_first + blockIdx.x;
+    if (u >= u_end) return;
+    int anc;
+    int64_t s, e, lo, hi;
+    unit_range(a.ut, u, &anc, &s, &e);
+    cand_range(a, s, &lo, &hi);
+    const int64_t n = hi - lo;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kIn = 8;
+    // per-head statistics over the candidates (k_stats): one warp per head
+    if (n > 0)
+        for (int h = warp; h < a.Hq; h += kTopkThreads / 32) {
+            const float* z = logits + (static_cast<int64_t>(u) * a.Hq + h) * a.nb;
+            float m = -INFINITY;
+            for (int64_t b0 = lo + lane; b0 < hi; b0 += 32 * kIn) {
+                float x[kIn];
+#pragma unroll
+                for (int i = 0; i < kIn; ++i) x[i] = b0 + 32 * i < hi ? z[b0 + 32 * i] : -INFINITY;
+#pragma unroll
+                for (int i = 0; i < kIn; ++i) m = fmaxf(m, x[i]);
+            }
+            for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
+            float sum = 0.f;
+            for (int64_t b0 = lo + lane; b0 < hi; b0 += 32 * kIn) {
+                float x[kIn];
+#pragma unroll
+                for (int i = 0; i < kIn; ++i) x[i] = b0 + 32 * i < hi ? z[b0 + 32 * i] : 0.f;
+#pragma unroll
+                for (int i = 0; i < kIn; ++i)
+                    if (b0 + 32 * i < hi) sum += expf(x[i] - m);
+            }
+            for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+            if (lane == 0) {
+                s_m[h] = m;
+                s_inv[h] = 1.0f / sum;
+            }
+        }
+    __syncthreads();
+    // soft vote over the heads in order (k_vote); the candidates' sort keys
+    int np = 1;
+    while (np < n) np <<= 1;
+    const bool sort = n > a.k;
+    for (int64_t b = threadIdx.x; b < a.nb; b += kTopkThreads) {
+        float score = __int_as_float(0x7FC00000);
+        if (b >= lo && b < hi) {
+            score = 0.f;
+            const float* zb = logits + static_cast<int64_t>(u) * a.Hq * a.nb + b;
+            for (int h0 = 0; h0 < a.Hq; h0 += kIn) {
+                float z[kIn], mx[kIn], inv[kIn];
+#pragma unroll
+                for (int i = 0; i < kIn; ++i) {
+                    const int h = h0 + i < a.Hq ? h0 + i : a.Hq - 1;
+                    z[i] = zb[static_cast<int64_t>(h) * a.nb];
+                    mx[i] = s_m[h];
+                    inv[i] = s_inv[h];
+                }
+#pragma unroll
+                for (int i = 0; i < kIn; ++i)
+                    if (h0 + i < a.Hq) score += expf(z[i] - mx[i]) * inv[i];
+            }
+            if (sort)
+                sk[b - lo] = (static_cast<uint64_t>(~float_key(score)) << 32) | static_cast<uint32_t>(b - lo);
+        }
+        scores[static_cast<int64_t>(u) * a.nb + b] = score;
+    }
+    int32_t* out = sel + static_cast<int64_t>(u) * a.k;
+    if (!sort) {
+        for (int i = threadIdx.x; i < a.k; i += blockDim.x) out[i] = (i < n) ? static_cast<int32_t>(lo + i) : -1;
+        if (threadIdx.x == 0) sel_count[u] = static_cast<int32_t>(n);
+        return;
+    }
+    for (int i = static_cast<int>(n) + threadIdx.x; i < np; i += kTopkThreads) sk[i] = ~0ull;  // padding sorts last
+    __syncthreads();
+    topk_sort_emit(sk, bm, np, lo, a.k, out);
+    if (threadIdx.x == 0) sel_count[u] = a.k;  // n > k: exactly k picks
 }
 
 // ---- top-k over many candidates per unit: the same radix select and ordered
@@ -891,6 +994,11 @@ cudaError_t launch_select(const Derived& d, int mode, int64_t tok_begin, int64_t
     if (e != cudaSuccess) return e;
     dim3 gl((max_units + upt - 1) / upt, static_cast<unsigned>((d.nb + 127) / 128), d.Hkv);
     k_logits<<<gl, kLtThreads, kLtSmem, st>>>(a, fingerprints, reps, logits);
+    if (d.nb <= kSortMax && d.Hq <= kFusedMaxHeads && d.k <= kSortMax) {
+        // every unit's candidates fit the sort: statistics, vote and top-k in one kernel
+        k_select_fused<<<max_units, kTopkThreads, 0, st>>>(a, logits, scores, sel_blocks, sel_count);
+        return cudaGetLastError();
+    }
     const int64_t rows = static_cast<int64_t>(max_units) * d.Hq;
     k_stats<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(a, logits, stats);
     k_vote<<<dim3(static_cast<unsigned>((d.nb + 255) / 256), max_units), 256, 0, st>>>(a, logits, stats, scores);

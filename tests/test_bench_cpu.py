@@ -67,15 +67,18 @@ def test_selection_agreement_counts():
 
 
 def test_launch_counts():
-    # step (a): k_block_reps, k_fingerprint, k_cluster (+ k_gram when clusters have > 1 sub-chunk)
-    assert bench.launches(workload("llama8b-128k"))["total"] == 9   # 4 + 4 + 1
-    assert bench.launches(workload("gqa4-4k", max_cluster_subchunks=1))["total"] == 8
+    # step (a): k_block_reps, k_fingerprint, k_cluster (+ k_gram when clusters have > 1 sub-chunk);
+    # selection: k_logits + k_select_fused (up to 4096 blocks); attention: k_sparse_attn
+    assert bench.launches(workload("llama8b-128k"))["total"] == 7   # 4 + 2 + 1
+    assert bench.launches(workload("gqa4-4k", max_cluster_subchunks=1))["total"] == 6
+    # more than 4096 blocks: k_logits, k_stats, k_vote, k_topk
+    assert bench.launches(workload("llama8b-1m", block_size=128))["total"] == 4 + 4 + 1
     # token level: split, two scoring passes and their merge, then the multi-CTA top-k
     # (init, 4 histogram passes, count, scan, emit)
     assert bench.launches(workload("llama8b-128k-tok"))["total"] == 3 + 4 + 8 + 3
     assert bench.launches(workload("llama8b-32k", block_size=1, top_k=1024))["total"] == 3 + 5 + 3
-    assert bench.launches(workload("llama8b-64k-32l"), 8)["total"] == 4 + 8 * 5
-    assert bench.launches(workload("llama8b-64k-32l"), 8, 8)["total"] == 8 * 4 + 8 * 5  # per-chunk step (a)
+    assert bench.launches(workload("llama8b-64k-32l"), 8)["total"] == 4 + 8 * 3
+    assert bench.launches(workload("llama8b-64k-32l"), 8, 8)["total"] == 8 * 4 + 8 * 3  # per-chunk step (a)
 
 
 def test_other_configs_compacts_each_side_run(monkeypatch):
