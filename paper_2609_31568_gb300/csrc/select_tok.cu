@@ -362,9 +362,9 @@ k_tok_score(const __grid_constant__ CUtensorMap tf, const __grid_constant__ CUte
 // pass 1 (NARROW) one CTA per 128 tokens (the votes are per token); with many
 // ranges the CTAs keep all KV heads and whole ranges, which amortises the
 // fingerprint loads and the pipeline start over more key tiles.
-constexpr int kNc = 16;
+constexpr int kNc = 16;                        // (unit, head) columns of a small tile
 constexpr int kRange1 = 128;                   // narrow pass 1: tokens per CTA
-constexpr int kFewRanges = 1024;               // below this many ranges: the split grids                        // (unit, head) columns of a small tile
+constexpr int kFewRanges = 1024;               // below this many ranges: the split grids
 constexpr uint32_t kFsHalf = 3 * kNc * 128;    // one 64-column half of the 48-row operand: 6 KB
 constexpr uint32_t kOffFs = 0;                 // fingerprint parts, 12 KB
 constexpr uint32_t kOffKs = 2 * kFsHalf;       // 2 key stages (a multiple of 1024)
