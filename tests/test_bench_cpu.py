@@ -77,6 +77,11 @@ def test_launch_counts():
     # (init, 4 histogram passes, count, scan, emit)
     assert bench.launches(workload("llama8b-128k-tok"))["total"] == 3 + 4 + 8 + 3
     assert bench.launches(workload("llama8b-32k", block_size=1, top_k=1024))["total"] == 3 + 5 + 3
+    # the 1M-token step of Algorithm 2: 16 outer chunks, one unit each (the ncu launch list of that step
+    # counted 288 launches of the library's kernels)
+    w = workload("llama8b-1m-tok")
+    chunks = w.n_tokens // w.outer_chunk
+    assert bench.launches(w, chunks, chunks)["total"] == 288
     assert bench.launches(workload("llama8b-64k-32l"), 8)["total"] == 4 + 8 * 3
     assert bench.launches(workload("llama8b-64k-32l"), 8, 8)["total"] == 8 * 4 + 8 * 3  # per-chunk step (a)
 
