@@ -345,7 +345,9 @@ int scale_prefill_host(const scale_params_t *p, int32_t mode, const void *q_host
 
 /* Upper bound, in nanoseconds of wall time, of every device-side wait of the
  * attention kernel (default 4e9). A wait that runs out records
- * SCALE_ERR_TIMEOUT in the device status and the kernel returns. Process-wide. */
+ * SCALE_ERR_TIMEOUT in the device status and the kernel returns. Process-wide;
+ * applies to launches issued after the call. ns = 0 is refused with
+ * SCALE_ERR_INVALID_ARG and leaves the limit unchanged. */
 int scale_set_wait_timeout_ns(uint64_t ns);
 
 /* Self-check of the bounded-wait machinery: launches one block that waits on an

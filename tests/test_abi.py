@@ -31,6 +31,14 @@ def test_every_declared_symbol_is_exported(lib):
     assert not missing
 
 
+def test_wait_limit_entry_points_validate(lib):
+    """A wait limit of 0 is refused and the default is accepted; the wait
+    self-check refuses a missing workspace before launching anything."""
+    assert lib.scale_set_wait_timeout_ns(0) == S.SCALE_ERR_INVALID_ARG
+    assert lib.scale_set_wait_timeout_ns(4_000_000_000) == S.SCALE_OK  # the default
+    assert lib.scale_selftest_wait_timeout(None, 0, 1_000_000, None) == S.SCALE_ERR_INVALID_ARG
+
+
 def test_params_struct_layout_matches_header():
     src = r"""
 #include <stddef.h>
